@@ -1,0 +1,411 @@
+"""Benchmark of the MT-DAO hot path on GB300.
+
+One benchmark "step" is one communication round of the workload: H local
+optimizer steps of all M replicas (H = the largest sync period), the round's
+due replica averages fused into its last step.  Default workload: the ~1B
+decoder-shaped parameter list (1,311,086,592 fp32 per replica, M=4, N=3,
+Adam, H=32), the configuration the bandwidth target is quoted on.
+
+Printed (rank 0, one JSON line): params/s = M * n * H / round time (whole
+job, all ranks), plus the roofline of the dominant kernel (the local-step
+kernel, timed per launch with CUDA events on its stream), the standalone
+sync kernel's bandwidth, an end-to-end figure through the host-buffer C-ABI
+call, and the CPU oracle timed on a bounded sample.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+                  [--workload decoder_1b|gpt2_small|decoder_350m|tiny]
+For N > 1 (torchrun) every rank runs its own independent replica set
+(weak scaling); only the timing is reduced across ranks.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+from synth import workloads as W  # noqa: E402
+
+PEAKS_FILE = os.path.join(ROOT, "MEASURED_PEAKS.json")
+TRAFFIC_FILE = os.path.join(ROOT, "profiles", "step_kernel_traffic.json")
+STEP_KERNEL_SRC = os.path.join(ROOT, "paper_2510_05361_gb300", "csrc", "step_kernels.cuh")
+FALLBACK_HBM_GBS = 6800.0
+L2_BYTES = 129 * 2 ** 20
+
+
+def parse_args():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=5)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", default="decoder_1b", choices=sorted(W.WORKLOADS))
+    ap.add_argument("--e2e-rounds", type=int, default=2)
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    return ap.parse_args()
+
+
+def round_len(opt) -> int:
+    periods = [opt["period_x"], opt.get("period_v", 0)] + list(opt["period_u"])
+    return max(p for p in periods if p > 0)
+
+
+def hbm_peak():
+    try:
+        with open(PEAKS_FILE) as f:
+            return float(json.load(f)["hbm_gbs"]), "measured"
+    except Exception:
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+def source_sha() -> str:
+    with open(STEP_KERNEL_SRC, "rb") as f:
+        return hashlib.sha256(f.read()).hexdigest()[:16]
+
+
+def measured_traffic(workload: str, per_launch_units: int):
+    """DRAM bytes per launch of the step kernel from the committed ncu
+    summary, scaled to this launch; None if absent or the kernel changed."""
+    try:
+        with open(TRAFFIC_FILE) as f:
+            rec = json.load(f)
+    except Exception:
+        return None
+    if rec.get("source_sha") != source_sha():
+        return None
+    per_unit = rec["dram_bytes"] / rec["elements"]
+    return int(round(per_unit * per_launch_units))
+
+
+# --------------------------------------------------------------------- clocks
+
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        try:
+            fd, self.path = tempfile.mkstemp(suffix=".csv")
+            os.close(fd)
+            self.out = open(self.path, "w")
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu), "--query-gpu=" + self.FIELDS,
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=self.out, stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+
+    def stop(self) -> dict:
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        self.out.close()
+        sm, smax, reasons, power = [], [], set(), []
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        with open(self.path) as f:
+            for line in f:
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) < 9:
+                    continue
+                try:
+                    sm.append(float(parts[1]))
+                    smax.append(float(parts[2]))
+                    power.append(float(parts[3]))
+                except ValueError:
+                    continue
+                for name, val in zip(names, parts[5:9]):
+                    if val.lower().startswith("active"):
+                        reasons.add(name)
+        os.unlink(self.path)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
+        loaded = [s for s, p in zip(sm, power) if p > 0.5 * max(power)] or sm
+        return {"sm_mhz": statistics.median(loaded), "sm_max_mhz": max(smax),
+                "reasons": sorted(reasons), "samples": len(sm),
+                "power_w_max": max(power)}
+
+
+# --------------------------------------------------------------------- CPU oracle
+
+def oracle_sample_rate(w, n_sample: int, rounds: int = 1):
+    """Time the CPU oracle (as it stands, one thread) on n_sample elements of
+    every replica for `rounds` rounds of H local steps with their syncs.
+    Returns (params/s, seconds, description)."""
+    import numpy as np
+
+    from oracle.oracle import Oracle
+    from synth import generators as G
+
+    lay = W.layout(w["shapes"])
+    opt, M = w["opt"], w["M"]
+    H = round_len(opt)
+    idx = np.arange(n_sample, dtype=np.int64)
+    x0 = G.init_params(w, lay, W.INIT_SEED, idx).astype(np.float64)
+    g = np.stack([G.grads(w, lay, W.GRAD_SEED, m, 0, idx) for m in range(M)]).astype(np.float64)
+    o = Oracle(opt, M, n_sample, x0=x0)
+    spent = 0.0
+    t = 0
+    for _ in range(rounds):
+        for _ in range(H):
+            t0 = time.perf_counter()
+            o.step(t, opt["lr"], g)
+            spent += time.perf_counter() - t0
+            t += 1
+    t0 = time.perf_counter()
+    o.settle(t)
+    spent += time.perf_counter() - t0
+    rate = M * n_sample * H * rounds / spent
+    desc = ("%d replicas x first %d elements x %d round(s) of %d local steps with the round's "
+            "syncs; one resident gradient batch" % (M, n_sample, rounds, H))
+    return rate, spent, desc
+
+
+def run_reference(args):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return 0
+    w = W.get(args.workload)
+    n_sample = 1 << 18
+    for _ in range(max(args.warmup, 0)):
+        oracle_sample_rate(w, n_sample)
+    rates, total = [], 0.0
+    for _ in range(args.steps):
+        r, s, desc = oracle_sample_rate(w, n_sample)
+        rates.append(r)
+        total += s
+    value = statistics.median(rates)
+    H = round_len(w["opt"])
+    line = {
+        "impl": "reference",
+        "metric": "fused MT-DAO step params/s (replica-parameter updates per second, syncs included)",
+        "value": value,
+        "unit": "params/s",
+        "n_gpus": args.gpus,
+        "steps": args.steps,
+        "warmup": args.warmup,
+        "ms_per_step": 1e3 * W.layout(w["shapes"])["n_padded"] * w["M"] * H / value,
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "f64",
+        "data": "synthetic",
+        "config": {"workload": w["name"], "desc": w["desc"], "sample": desc},
+        "cpu_baseline": {"value": value, "unit": "params/s", "cores": 1, "kind": "oracle",
+                         "sample": desc},
+        "e2e": {"value": value, "unit": "params/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+        "gpu_launches": 0,
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+# --------------------------------------------------------------------- GPU arm
+
+def run_ours(args):
+    import torch
+
+    import paper_2510_05361_gb300 as P
+    from synth.device import DeviceInputs
+
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    P.load()
+
+    w = W.get(args.workload)
+    opt, M = w["opt"], w["M"]
+    lay = W.layout(w["shapes"])
+    n = lay["n_padded"]
+    H = round_len(opt)
+    gdt = P.BF16 if w["grad_dtype"] == "bf16" else P.F32
+    g_bytes = 2 if gdt == P.BF16 else 4
+    n_states = 1 + opt["n_mom"] + (0 if opt["base"] == "sgdm" else 1)
+    step_bytes = W.bytes_per_step(w)
+    stream = torch.cuda.current_stream()
+
+    eng = P.MTDAO(opt, M, w["shapes"], stream=stream.cuda_stream)
+    inputs = DeviceInputs(w, lay, W.GRAD_SEED, W.INIT_SEED)
+    eng.set_params(inputs.init_params())
+    grads = inputs.grads(0)            # one resident batch, reused every local step
+    torch.cuda.synchronize()
+
+    small = step_bytes < 8 * L2_BYTES
+    flush = torch.empty(2 * L2_BYTES // 4, dtype=torch.float32, device="cuda") if small else None
+
+    def one_round(events=None):
+        for k in range(H):
+            mask = eng.sync_due()
+            if flush is not None:
+                flush.fill_(1.0)
+            if events is not None:
+                events[k][0].record(stream)
+            P.mtdao_step(eng.h, grads.data_ptr(), gdt, opt["lr"], mask)
+            if events is not None:
+                events[k][1].record(stream)
+
+    for _ in range(args.warmup):
+        one_round()
+    torch.cuda.synchronize()
+
+    sampler = ClockSampler(local)
+    if dist is not None:
+        dist.barrier()
+    torch.cuda.synchronize()
+    sampler.start()
+    time.sleep(0.3)
+    rounds_ev = [[(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+                  for _ in range(H)] for _ in range(args.steps)]
+    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    start.record(stream)
+    for r in range(args.steps):
+        one_round(rounds_ev[r])
+    end.record(stream)
+    torch.cuda.synchronize()
+    if dist is not None:
+        dist.barrier()
+    clocks = sampler.stop()
+    elapsed_ms = start.elapsed_time(end)
+    launch_ms = [[a.elapsed_time(b) for a, b in rnd] for rnd in rounds_ev]
+    plain = [ms for rnd in launch_ms for ms in rnd[:-1]] or [ms for rnd in launch_ms for ms in rnd]
+    sync_steps = [rnd[-1] for rnd in launch_ms]
+    if small:
+        # L2 was flushed before every launch; time only the launches.
+        elapsed_ms = sum(ms for rnd in launch_ms for ms in rnd)
+    if dist is not None:
+        t = torch.tensor([elapsed_ms], device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        elapsed_ms = float(t.item())
+
+    units = world * M * n * H * args.steps
+    value = units / (elapsed_ms / 1e3)
+    step_ms = statistics.mean(plain)
+    peak, peak_kind = hbm_peak()
+    achieved = step_bytes / (step_ms / 1e3) / 1e9
+
+    # standalone replica-average kernel (all states), timed separately
+    sync_ms = []
+    all_mask = (1 << n_states) - 1
+    for i in range(6):
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        if flush is not None:
+            flush.fill_(1.0)
+        a.record(stream)
+        P.mtdao_sync(eng.h, all_mask)
+        b.record(stream)
+        torch.cuda.synchronize()
+        if i >= 2:
+            sync_ms.append(a.elapsed_time(b))
+    sync_bytes = W.bytes_per_sync(w, n_states)
+    sync_gbs = sync_bytes / (statistics.median(sync_ms) / 1e3) / 1e9
+
+    # end to end through the host-buffer C-ABI call
+    e2e = None
+    if not args.no_e2e and args.e2e_rounds > 0:
+        host_g = torch.empty((M, n), dtype=grads.dtype, pin_memory=True)
+        host_g.copy_(grads)
+        host_x = torch.empty((n,), dtype=torch.float32, pin_memory=True)
+        P.mtdao_step_host(eng.h, host_g.data_ptr(), gdt, opt["lr"], eng.sync_due())
+        torch.cuda.synchronize()
+        if dist is not None:
+            dist.barrier()
+        t0 = time.perf_counter()
+        for _ in range(args.e2e_rounds):
+            for _ in range(H):
+                P.mtdao_step_host(eng.h, host_g.data_ptr(), gdt, opt["lr"], eng.sync_due())
+            P.mtdao_copy_state_to_host(eng.h, 0, 0, host_x.data_ptr())   # round's synced x
+        torch.cuda.synchronize()
+        e2e_s = time.perf_counter() - t0
+        if dist is not None:
+            t = torch.tensor([e2e_s], device="cuda")
+            dist.all_reduce(t, op=dist.ReduceOp.MAX)
+            e2e_s = float(t.item())
+        e2e = {"value": world * M * n * H * args.e2e_rounds / e2e_s, "unit": "params/s",
+               "h2d_bytes_per_step": H * M * n * g_bytes, "d2h_bytes_per_step": n * 4,
+               "rounds": args.e2e_rounds}
+        del host_g
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        rate, spent, desc = oracle_sample_rate(w, 1 << 20)
+        cpu = {"value": rate, "unit": "params/s", "cores": 1, "kind": "oracle", "sample": desc,
+               "seconds": round(spent, 2)}
+
+    traffic = measured_traffic(w["name"], M * n)
+    line = {
+        "metric": "fused MT-DAO step params/s (replica-parameter updates per second, syncs included)",
+        "value": value,
+        "unit": "params/s",
+        "n_gpus": world,
+        "steps": args.steps,
+        "warmup": args.warmup,
+        "ms_per_step": elapsed_ms / args.steps,
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "f32",
+        "data": "synthetic",
+        "config": {
+            "workload": w["name"], "desc": w["desc"], "M": M, "n_padded": n, "n_mom": opt["n_mom"],
+            "base": opt["base"], "grad_dtype": w["grad_dtype"], "local_steps_per_step": H,
+            "step": "one communication round: H local steps, the due averages fused into the last",
+            "grads": "one resident synthetic gradient batch per replica, reused every local step",
+            "l2": ("L2 flushed before every launch; time = sum of launch times" if small else
+                   "inputs larger than L2 (%.0f GB resident)" % ((n_states * 4 + g_bytes) * M * n / 1e9)),
+            "parallelism": "replicas only" if world == 1 else "independent replica set per GPU",
+        },
+        "step_kernel": {"ms_mean": step_ms, "ms_min": min(plain), "bytes": step_bytes,
+                        "gbs": achieved, "params_per_s": M * n / (step_ms / 1e3)},
+        "sync_step_kernel": {"ms_mean": statistics.mean(sync_steps),
+                             "gbs": step_bytes / (statistics.mean(sync_steps) / 1e3) / 1e9},
+        "sync_kernel": {"ms_median": statistics.median(sync_ms), "bytes": sync_bytes, "gbs": sync_gbs,
+                        "frac": sync_gbs / peak, "states": n_states},
+        "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+                     "frac": achieved / peak, "traffic": traffic, "peak_kind": peak_kind,
+                     "kernel": "step_kernel (local step, no sync)"},
+        "cpu_baseline": cpu,
+        "e2e": e2e,
+        "gpu_launches": args.steps * H * (3 if opt.get("clip_mode") == "global_norm" else 1),
+        "clocks": clocks,
+    }
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    eng.close()
+    if dist is not None:
+        dist.destroy_process_group()
+    return 0
+
+
+def main():
+    args = parse_args()
+    if args.impl == "reference":
+        return run_reference(args)
+    return run_ours(args)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

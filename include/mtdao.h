@@ -1,0 +1,270 @@
+/*
+ * mtdao.h -- C ABI of the GB300 MT-DAO hot path (libmtdao.so).
+ *
+ * MT-DAO (Multi-timescale Distributed Adaptive Optimizers, arXiv 2510.05361)
+ * runs M data-parallel workers that each take local optimizer steps with N
+ * first-momentum EMAs at different beta timescales (section 2.3, Algorithm 1
+ * for Adam, Algorithm 2 for ADOPT, Algorithm 3 for SGDM) and periodically
+ * average their parameters x, each momentum u^j and the second moment v over
+ * the workers, every state on its own period K_x, K_j, K_v.  This library
+ * keeps the M workers as M replicas resident in one GPU's memory: the local
+ * step is one fused elementwise pass over HBM and the averaging is an
+ * in-memory reduction across replicas.
+ *
+ * Conventions shared by every call
+ *   - Status: every call returns an mtdao_status (0 = success, negative =
+ *     error) unless stated otherwise; nothing is thrown across the ABI.  The
+ *     message of the last failure is kept per handle (mtdao_last_error).
+ *   - Streams: all device work is enqueued on the handle's CUDA stream and is
+ *     asynchronous unless a call says it synchronises.  Pointers marked
+ *     "device" must be device-accessible on the handle's device.
+ *   - Ownership: the library owns the state arena (x, u^1..u^N, v for all
+ *     replicas) and its workspaces; the caller owns gradients, output buffers
+ *     and the stream.
+ *   - Threads: a handle must not be used from two threads at once.
+ *   - Layout: the caller's list of tensors (numel_k, k = 0..n_tensors-1) is
+ *     flattened into one per-replica vector of n_padded fp32 elements.
+ *     Tensor k starts at offset_k, a multiple of 8 elements; padding between
+ *     tensors and at the end is zero and stays zero when the gradient's
+ *     padding is zero.  n_padded is a multiple of 256 elements.  State s of
+ *     replica m occupies arena[(s*M + m)*n_padded .. +n_padded).
+ *   - States: index 0 = x, 1..N = u^1..u^N, N+1 = v (Adam and ADOPT only).
+ *     A sync mask has bit s set for state s.
+ *   - Numerics: states are fp32; every update is computed in fp32 with
+ *     IEEE-rounded division and square root (no fast-math).  Per-step
+ *     scalars (bias corrections, clip bounds) are computed in double on the
+ *     host and rounded once.
+ */
+#ifndef MTDAO_H
+#define MTDAO_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define MTDAO_VERSION 1
+#define MTDAO_MAX_MOM 4          /* largest N supported */
+#define MTDAO_MAX_REPLICAS 64    /* largest M supported */
+
+typedef enum {
+    MTDAO_OK = 0,
+    MTDAO_ERR_INVALID = -1,      /* bad argument or configuration */
+    MTDAO_ERR_OOM = -2,          /* device or pinned-host allocation failed */
+    MTDAO_ERR_CUDA = -3,         /* a CUDA runtime call or launch failed */
+    MTDAO_ERR_ALIGN = -4,        /* a pointer is not 16-byte aligned */
+    MTDAO_ERR_STATE = -5         /* call not allowed in the handle's state */
+} mtdao_status;
+
+typedef enum {
+    MTDAO_BASE_ADAM = 0,         /* Algorithm 1 */
+    MTDAO_BASE_ADOPT = 1,        /* Algorithm 2 */
+    MTDAO_BASE_SGDM = 2          /* Algorithm 3 */
+} mtdao_base;
+
+typedef enum {
+    MTDAO_CLIP_NONE = 0,
+    /* Adam/SGDM clip(g, rho): each replica's whole flattened gradient is
+     * scaled by min(1, rho / (||g||_2 + 1e-6)); v keeps the raw gradient. */
+    MTDAO_CLIP_GLOBAL_NORM = 1,
+    /* ADOPT clip(g-hat, c_t): elementwise clamp to +-c_t, c_t = (t+1)^(1/4). */
+    MTDAO_CLIP_ELEMENTWISE = 2
+} mtdao_clip;
+
+typedef enum { MTDAO_F32 = 0, MTDAO_BF16 = 1 } mtdao_dtype;
+
+typedef enum {
+    /* Algorithm 1: a state whose period K divides the completed local-step
+     * count c = t+1 is averaged at the end of step t. */
+    MTDAO_PHASE_ALG1 = 0,
+    /* Algorithm 2 as printed: u^j and v are averaged at the end of step t
+     * when t mod K == 0, x when (t+1) mod K_x == 0. */
+    MTDAO_PHASE_ALG2_LITERAL = 1
+} mtdao_phase;
+
+/*
+ * Hyper-parameters of Algorithms 1-3 (their "Require" lists).  Decay rates
+ * and weights are doubles so that 1 - beta keeps its precision.
+ */
+typedef struct {
+    int32_t base;                       /* mtdao_base */
+    int32_t n_mom;                      /* N, 1..MTDAO_MAX_MOM */
+    double beta1[MTDAO_MAX_MOM];        /* beta_{1,j} in [0, 1) */
+    double omega[MTDAO_MAX_MOM];        /* omega_j in [0, 1], sum <= 1 */
+    double beta2;                       /* beta_2 in [0, 1) (Adam, ADOPT) */
+    double eps;                         /* epsilon > 0 (Adam, ADOPT) */
+    int32_t bias_correction;            /* Adam: 1 = divide u^j by 1-beta_{1,j}^(t+1)
+                                           and v by 1-beta_2^(t+1); 0 = Algorithm 1
+                                           as printed.  Must be 0 otherwise. */
+    int32_t clip_mode;                  /* mtdao_clip */
+    double clip_rho;                    /* rho > 0 for MTDAO_CLIP_GLOBAL_NORM */
+    int32_t sync_phase;                 /* mtdao_phase */
+    int64_t period_x;                   /* K_x; 0 = never averaged */
+    int64_t period_u[MTDAO_MAX_MOM];    /* K_j; 0 = never */
+    int64_t period_v;                   /* K_v; 0 = never (ignored for SGDM) */
+} mtdao_config;
+
+typedef struct mtdao_ctx *mtdao_handle;
+
+/* ------------------------------------------------------------------ host-only */
+
+/* MTDAO_VERSION of the loaded library. */
+int32_t mtdao_version(void);
+
+/*
+ * Fill *cfg with defaults for a base and N: beta_1 = (0.9, 0.999, 0.5, 0.99)
+ * prefix, omega_j = 0.95/N, beta_2 = 0.999 (0.9999 for ADOPT, section 4.1),
+ * eps = 1e-8, bias correction on for Adam, no clipping, Algorithm 1 phase,
+ * all periods 32 (section 4.1 default K).  No device access.
+ */
+int mtdao_config_default(mtdao_config *cfg, int32_t base, int32_t n_mom);
+
+/*
+ * Check a configuration for M replicas against the ranges of Algorithms
+ * 1-3 (beta in [0,1), omega_j in [0,1], sum omega <= 1 + 1e-6, periods >= 0,
+ * clip mode matching the base).  MTDAO_OK or MTDAO_ERR_INVALID; the reason
+ * is available from mtdao_last_error(NULL).  No device access.
+ */
+int mtdao_config_validate(const mtdao_config *cfg, int32_t M);
+
+/* Number of state vectors per replica: 1 + N (+1 for v unless SGDM). */
+int32_t mtdao_num_states(const mtdao_config *cfg);
+
+/*
+ * Flattened layout of a tensor list: offsets_out[k] (n_tensors entries,
+ * caller-owned) and *n_padded_out as described under "Layout" above.
+ * MTDAO_ERR_INVALID for a non-positive numel or n_tensors.  No device access.
+ */
+int mtdao_plan_layout(const int64_t *tensor_numel, int32_t n_tensors,
+                      int64_t *offsets_out, int64_t *n_padded_out);
+
+/*
+ * Sync schedule (Algorithms 1 and 2, the "sync every K steps" rows): the
+ * mask of states to average at the end of local step `step` (0-based)
+ * under cfg->sync_phase.  No device access.
+ */
+int mtdao_due_mask(const mtdao_config *cfg, int64_t step, uint32_t *mask_out);
+
+/* ------------------------------------------------------------------ lifecycle */
+
+/*
+ * Create a handle on the current CUDA device for M replicas of the tensor
+ * list tensor_numel[0..n_tensors-1] (host array).  Allocates the state
+ * arena (num_states * M * n_padded fp32) and workspaces, zeroes every state
+ * and sets the step counter t to 0.  cuda_stream is a cudaStream_t (NULL =
+ * legacy default stream).  On failure *out is NULL and the reason is
+ * available from mtdao_last_error(NULL).  Synchronises the stream once.
+ */
+int mtdao_create(const mtdao_config *cfg, int32_t M, const int64_t *tensor_numel,
+                 int32_t n_tensors, void *cuda_stream, mtdao_handle *out);
+
+/* Release everything the handle owns.  NULL-safe.  Synchronises its streams. */
+void mtdao_destroy(mtdao_handle h);
+
+/* Switch the stream later calls enqueue on (the caller orders the change). */
+int mtdao_set_stream(mtdao_handle h, void *cuda_stream);
+
+/*
+ * Initial state (Algorithm 1 "for each worker: initialize"): copy x0
+ * (device, [n_padded] fp32, padding zero) into x of every replica, zero all
+ * u^j and v, set t = 0.  All workers start from the same x_0 (appendix,
+ * x_{-1} = x_0 shared).
+ */
+int mtdao_set_params(mtdao_handle h, const float *x0_dev);
+
+/* ------------------------------------------------------------------ hot path */
+
+/*
+ * One local step t (= the handle's counter, then t+1) of Algorithm 1, 2 or 3
+ * on every replica, as one pass over HBM:
+ *   Adam  : g-hat = clip(g); u^j = beta_j u^j + (1-beta_j) g-hat;
+ *           v = beta_2 v + (1-beta_2) g^2;
+ *           Delta = [(1-sum w) g-hat + sum w_j u^j/b_j] / (sqrt(v/b_v) + eps);
+ *           x = x - lr * Delta        (b = 1 - beta^(t+1), or 1 if no correction)
+ *   ADOPT : v = beta_2 v + (1-beta_2) g^2; g-tilde = clip(g/(sqrt(v)+eps), c_t);
+ *           u^j = beta_j u^j + (1-beta_j) g-tilde;
+ *           Delta = (1-sum w) g-tilde + sum w_j u^j;  x = x - lr * Delta
+ *   SGDM  : as Adam without v and without the denominator.
+ * grads_dev: device, [M][n_padded] of grad_dtype (mtdao_dtype), 16-byte
+ *   aligned, padding zero; read only.
+ * lr: eta_t for this step.
+ * sync_mask: states to average over the replicas at the end of this same
+ *   step (E_m[.] of Algorithm 1); usually the value of mtdao_sync_due.  The
+ *   average is fused into the step's pass: it costs no extra HBM traffic for
+ *   M in {2, 4, 8}; other M fall back to a separate averaging pass.
+ * With MTDAO_CLIP_GLOBAL_NORM a reduction pass over grads precedes the step.
+ * Errors: MTDAO_ERR_INVALID (dtype, mask bits beyond the states),
+ * MTDAO_ERR_ALIGN, MTDAO_ERR_CUDA.  On error t is unchanged.
+ */
+int mtdao_step(mtdao_handle h, const void *grads_dev, int32_t grad_dtype, double lr,
+               uint32_t sync_mask);
+
+/*
+ * mtdao_step with the gradients in host memory: they are copied to a
+ * library-owned device staging buffer (allocated on first use, two buffers
+ * so that a copy can overlap the previous step) and the step runs from
+ * there.  grads_host should be pinned for the copy to be asynchronous; it
+ * must stay unchanged until the call's work on the stream has completed.
+ */
+int mtdao_step_host(mtdao_handle h, const void *grads_host, int32_t grad_dtype, double lr,
+                    uint32_t sync_mask);
+
+/*
+ * Outer synchronisation (Algorithms 1-3, E_m[.] with OuterOpt = averaging):
+ * every state in mask is replaced, on every replica, by the equal-weight
+ * mean over the M replicas.  Computed as s_0 + (sum_m (s_m - s_0)) / M in
+ * fp32, which returns s_0 exactly when the replicas agree.  mask 0 is a no-op.
+ */
+int mtdao_sync(mtdao_handle h, uint32_t mask);
+
+/* Mask of states due at the end of the next step (mtdao_due_mask at t). */
+int mtdao_sync_due(mtdao_handle h, uint32_t *mask_out);
+
+/*
+ * Squared L2 norm of each replica's flattened gradient (the quantity that
+ * clip(g, rho) of Algorithms 1 and 3 is based on): out_dev (device, M
+ * doubles, caller-owned) receives sum_i g[m][i]^2.  Deterministic: fixed
+ * grid and fixed reduction order.  Uses a handle-owned workspace of partial
+ * sums.
+ */
+int mtdao_grad_sqnorm(mtdao_handle h, const void *grads_dev, int32_t grad_dtype,
+                      double *out_dev);
+
+/* ------------------------------------------------------------------ state access */
+
+/* Device pointer to state `state` of replica `replica` ([n_padded] fp32). */
+int mtdao_get_state_ptr(mtdao_handle h, int32_t state, int32_t replica, float **dev_ptr);
+
+/* Copy one state vector to host memory ([n_padded] floats); synchronises. */
+int mtdao_copy_state_to_host(mtdao_handle h, int32_t state, int32_t replica, float *host_out);
+
+/* Copy one state vector from host memory ([n_padded] floats); synchronises. */
+int mtdao_copy_state_from_host(mtdao_handle h, int32_t state, int32_t replica,
+                               const float *host_in);
+
+/*
+ * Layout of the handle: *n_padded, *n_tensors, *M, *n_states and a pointer
+ * to the handle-owned offsets array (valid until destroy).  Any output
+ * pointer may be NULL.
+ */
+int mtdao_layout(mtdao_handle h, int64_t *n_padded, int32_t *n_tensors, int32_t *M,
+                 int32_t *n_states, const int64_t **tensor_offsets);
+
+/* Step counter t (local steps taken); -1 for a NULL handle. */
+int64_t mtdao_get_step(mtdao_handle h);
+
+/* Set t, e.g. when resuming from a checkpoint of the states; t >= 0. */
+int mtdao_set_step(mtdao_handle h, int64_t step);
+
+/*
+ * Message of the handle's last failure ("" if none).  With h == NULL: the
+ * last failure of mtdao_create / mtdao_config_validate in this thread.
+ */
+const char *mtdao_last_error(mtdao_handle h);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* MTDAO_H */

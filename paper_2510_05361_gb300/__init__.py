@@ -1,0 +1,361 @@
+"""GB300-native MT-DAO hot path: Python binding of ``libmtdao.so``.
+
+Thin ctypes marshalling over the C ABI declared in ``include/mtdao.h``; the
+functions keep the C names (``mtdao_create``, ``mtdao_step``, ``mtdao_sync``,
+``mtdao_destroy``, ...).  Every step of the optimizer runs in the library's
+CUDA kernels; this module only converts arguments.  PyTorch is used by
+callers for device memory and streams.
+
+The library is loaded on first use; if it has not been built (see
+``paper_2510_05361_gb300.build``) that first use raises instead of falling
+back to anything else.  ``load()`` forces the load.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+from .build import LIB as _LIB_PATH
+
+MAX_MOM = 4
+MAX_REPLICAS = 64
+
+OK, ERR_INVALID, ERR_OOM, ERR_CUDA, ERR_ALIGN, ERR_STATE = 0, -1, -2, -3, -4, -5
+BASE_ADAM, BASE_ADOPT, BASE_SGDM = 0, 1, 2
+CLIP_NONE, CLIP_GLOBAL_NORM, CLIP_ELEMENTWISE = 0, 1, 2
+F32, BF16 = 0, 1
+PHASE_ALG1, PHASE_ALG2_LITERAL = 0, 1
+
+BASES = {"adam": BASE_ADAM, "adopt": BASE_ADOPT, "sgdm": BASE_SGDM}
+CLIPS = {"none": CLIP_NONE, "global_norm": CLIP_GLOBAL_NORM, "elementwise": CLIP_ELEMENTWISE}
+PHASES = {"alg1": PHASE_ALG1, "alg2_literal": PHASE_ALG2_LITERAL}
+DTYPES = {"f32": F32, "bf16": BF16}
+
+
+class mtdao_config(ctypes.Structure):
+    _fields_ = [
+        ("base", ctypes.c_int32),
+        ("n_mom", ctypes.c_int32),
+        ("beta1", ctypes.c_double * MAX_MOM),
+        ("omega", ctypes.c_double * MAX_MOM),
+        ("beta2", ctypes.c_double),
+        ("eps", ctypes.c_double),
+        ("bias_correction", ctypes.c_int32),
+        ("clip_mode", ctypes.c_int32),
+        ("clip_rho", ctypes.c_double),
+        ("sync_phase", ctypes.c_int32),
+        ("period_x", ctypes.c_int64),
+        ("period_u", ctypes.c_int64 * MAX_MOM),
+        ("period_v", ctypes.c_int64),
+    ]
+
+
+class MTDAOError(RuntimeError):
+    def __init__(self, code, msg):
+        super().__init__("mtdao error %d: %s" % (code, msg))
+        self.code = code
+
+
+def _load():
+    if not os.path.exists(_LIB_PATH):
+        raise ImportError("libmtdao.so is not built (%s); run "
+                          "`python -m paper_2510_05361_gb300.build`" % _LIB_PATH)
+    lib = ctypes.CDLL(_LIB_PATH)
+    H = ctypes.c_void_p
+    cfgp = ctypes.POINTER(mtdao_config)
+    i64p = ctypes.POINTER(ctypes.c_int64)
+    sig = {
+        "mtdao_version": (ctypes.c_int32, []),
+        "mtdao_config_default": (ctypes.c_int, [cfgp, ctypes.c_int32, ctypes.c_int32]),
+        "mtdao_config_validate": (ctypes.c_int, [cfgp, ctypes.c_int32]),
+        "mtdao_num_states": (ctypes.c_int32, [cfgp]),
+        "mtdao_plan_layout": (ctypes.c_int, [i64p, ctypes.c_int32, i64p, i64p]),
+        "mtdao_due_mask": (ctypes.c_int, [cfgp, ctypes.c_int64, ctypes.POINTER(ctypes.c_uint32)]),
+        "mtdao_create": (ctypes.c_int, [cfgp, ctypes.c_int32, i64p, ctypes.c_int32, ctypes.c_void_p,
+                                        ctypes.POINTER(H)]),
+        "mtdao_destroy": (None, [H]),
+        "mtdao_set_stream": (ctypes.c_int, [H, ctypes.c_void_p]),
+        "mtdao_set_params": (ctypes.c_int, [H, ctypes.c_void_p]),
+        "mtdao_step": (ctypes.c_int, [H, ctypes.c_void_p, ctypes.c_int32, ctypes.c_double,
+                                      ctypes.c_uint32]),
+        "mtdao_step_host": (ctypes.c_int, [H, ctypes.c_void_p, ctypes.c_int32, ctypes.c_double,
+                                           ctypes.c_uint32]),
+        "mtdao_sync": (ctypes.c_int, [H, ctypes.c_uint32]),
+        "mtdao_sync_due": (ctypes.c_int, [H, ctypes.POINTER(ctypes.c_uint32)]),
+        "mtdao_grad_sqnorm": (ctypes.c_int, [H, ctypes.c_void_p, ctypes.c_int32, ctypes.c_void_p]),
+        "mtdao_get_state_ptr": (ctypes.c_int, [H, ctypes.c_int32, ctypes.c_int32,
+                                               ctypes.POINTER(ctypes.c_void_p)]),
+        "mtdao_copy_state_to_host": (ctypes.c_int, [H, ctypes.c_int32, ctypes.c_int32, ctypes.c_void_p]),
+        "mtdao_copy_state_from_host": (ctypes.c_int, [H, ctypes.c_int32, ctypes.c_int32,
+                                                      ctypes.c_void_p]),
+        "mtdao_layout": (ctypes.c_int, [H, i64p, ctypes.POINTER(ctypes.c_int32),
+                                        ctypes.POINTER(ctypes.c_int32), ctypes.POINTER(ctypes.c_int32),
+                                        ctypes.POINTER(i64p)]),
+        "mtdao_get_step": (ctypes.c_int64, [H]),
+        "mtdao_set_step": (ctypes.c_int, [H, ctypes.c_int64]),
+        "mtdao_last_error": (ctypes.c_char_p, [H]),
+    }
+    for name, (res, args) in sig.items():
+        f = getattr(lib, name)
+        f.restype = res
+        f.argtypes = args
+    return lib
+
+
+class _LazyLib:
+    """Loads libmtdao.so on first attribute access."""
+
+    _handle = None
+
+    def __getattr__(self, name):
+        if _LazyLib._handle is None:
+            _LazyLib._handle = _load()
+        return getattr(_LazyLib._handle, name)
+
+
+lib = _LazyLib()
+LIB_PATH = _LIB_PATH
+
+
+def load():
+    """Load libmtdao.so now (raises ImportError if it is not built)."""
+    return lib.mtdao_version()
+
+
+def _check(rc, h=None):
+    if rc != OK:
+        raise MTDAOError(rc, (lib.mtdao_last_error(h) or b"").decode())
+    return rc
+
+
+def make_config(opt: dict) -> mtdao_config:
+    """mtdao_config from a plain dictionary (base, n_mom, beta1, omega, ...)."""
+    c = mtdao_config()
+    n = int(opt["n_mom"])
+    c.base = BASES[opt["base"]] if isinstance(opt["base"], str) else int(opt["base"])
+    c.n_mom = n
+    for j in range(n):
+        c.beta1[j] = float(opt["beta1"][j])
+        c.omega[j] = float(opt["omega"][j])
+        c.period_u[j] = int(opt["period_u"][j])
+    c.beta2 = float(opt.get("beta2", 0.999))
+    c.eps = float(opt.get("eps", 1e-8))
+    c.bias_correction = 1 if opt.get("bias_correction", c.base == BASE_ADAM) else 0
+    c.clip_mode = CLIPS[opt.get("clip_mode", "none")]
+    c.clip_rho = float(opt.get("clip_rho", 1.0))
+    c.sync_phase = PHASES[opt.get("sync_phase", "alg1")]
+    c.period_x = int(opt["period_x"])
+    c.period_v = int(opt.get("period_v", 0))
+    return c
+
+
+# ---- same-name wrappers of the C ABI (argument marshalling only) ----------
+
+def mtdao_version() -> int:
+    return int(lib.mtdao_version())
+
+
+def mtdao_config_default(base: int, n_mom: int) -> mtdao_config:
+    c = mtdao_config()
+    _check(lib.mtdao_config_default(ctypes.byref(c), base, n_mom))
+    return c
+
+
+def mtdao_config_validate(cfg: mtdao_config, M: int) -> None:
+    _check(lib.mtdao_config_validate(ctypes.byref(cfg), M))
+
+
+def mtdao_num_states(cfg: mtdao_config) -> int:
+    return int(lib.mtdao_num_states(ctypes.byref(cfg)))
+
+
+def mtdao_plan_layout(numels):
+    n = len(numels)
+    arr = (ctypes.c_int64 * n)(*[int(k) for k in numels])
+    offs = (ctypes.c_int64 * n)()
+    npad = ctypes.c_int64()
+    _check(lib.mtdao_plan_layout(arr, n, offs, ctypes.byref(npad)))
+    return list(offs), int(npad.value)
+
+
+def mtdao_due_mask(cfg: mtdao_config, step: int) -> int:
+    m = ctypes.c_uint32()
+    _check(lib.mtdao_due_mask(ctypes.byref(cfg), int(step), ctypes.byref(m)))
+    return int(m.value)
+
+
+def mtdao_create(cfg: mtdao_config, M: int, numels, stream: int = 0):
+    n = len(numels)
+    arr = (ctypes.c_int64 * n)(*[int(k) for k in numels])
+    h = ctypes.c_void_p()
+    _check(lib.mtdao_create(ctypes.byref(cfg), M, arr, n, ctypes.c_void_p(stream), ctypes.byref(h)))
+    return h
+
+
+def mtdao_destroy(h) -> None:
+    lib.mtdao_destroy(h)
+
+
+def mtdao_set_stream(h, stream: int) -> None:
+    _check(lib.mtdao_set_stream(h, ctypes.c_void_p(stream)), h)
+
+
+def mtdao_set_params(h, x0_dev_ptr: int) -> None:
+    _check(lib.mtdao_set_params(h, ctypes.c_void_p(x0_dev_ptr)), h)
+
+
+def mtdao_step(h, grads_dev_ptr: int, grad_dtype: int, lr: float, sync_mask: int = 0) -> None:
+    _check(lib.mtdao_step(h, ctypes.c_void_p(grads_dev_ptr), grad_dtype, float(lr), sync_mask), h)
+
+
+def mtdao_step_host(h, grads_host_ptr: int, grad_dtype: int, lr: float, sync_mask: int = 0) -> None:
+    _check(lib.mtdao_step_host(h, ctypes.c_void_p(grads_host_ptr), grad_dtype, float(lr), sync_mask), h)
+
+
+def mtdao_sync(h, mask: int) -> None:
+    _check(lib.mtdao_sync(h, mask), h)
+
+
+def mtdao_sync_due(h) -> int:
+    m = ctypes.c_uint32()
+    _check(lib.mtdao_sync_due(h, ctypes.byref(m)), h)
+    return int(m.value)
+
+
+def mtdao_grad_sqnorm(h, grads_dev_ptr: int, grad_dtype: int, out_dev_ptr: int) -> None:
+    _check(lib.mtdao_grad_sqnorm(h, ctypes.c_void_p(grads_dev_ptr), grad_dtype,
+                                 ctypes.c_void_p(out_dev_ptr)), h)
+
+
+def mtdao_get_state_ptr(h, state: int, replica: int) -> int:
+    p = ctypes.c_void_p()
+    _check(lib.mtdao_get_state_ptr(h, state, replica, ctypes.byref(p)), h)
+    return int(p.value)
+
+
+def mtdao_copy_state_to_host(h, state: int, replica: int, host_ptr: int) -> None:
+    _check(lib.mtdao_copy_state_to_host(h, state, replica, ctypes.c_void_p(host_ptr)), h)
+
+
+def mtdao_copy_state_from_host(h, state: int, replica: int, host_ptr: int) -> None:
+    _check(lib.mtdao_copy_state_from_host(h, state, replica, ctypes.c_void_p(host_ptr)), h)
+
+
+def mtdao_layout(h) -> dict:
+    npad, nt, M, ns = ctypes.c_int64(), ctypes.c_int32(), ctypes.c_int32(), ctypes.c_int32()
+    offs = ctypes.POINTER(ctypes.c_int64)()
+    _check(lib.mtdao_layout(h, ctypes.byref(npad), ctypes.byref(nt), ctypes.byref(M), ctypes.byref(ns),
+                            ctypes.byref(offs)), h)
+    return {"n_padded": int(npad.value), "n_tensors": int(nt.value), "M": int(M.value),
+            "n_states": int(ns.value), "offsets": [int(offs[i]) for i in range(nt.value)]}
+
+
+def mtdao_get_step(h) -> int:
+    return int(lib.mtdao_get_step(h))
+
+
+def mtdao_set_step(h, step: int) -> None:
+    _check(lib.mtdao_set_step(h, int(step)), h)
+
+
+def mtdao_last_error(h=None) -> str:
+    return (lib.mtdao_last_error(h) or b"").decode()
+
+
+class MTDAO:
+    """Owning wrapper of one handle: M replicas of a flattened tensor list.
+
+    ``opt`` is a plain dictionary (see ``make_config``).  Device buffers are
+    passed as torch tensors or raw pointers; the stream is torch's current
+    stream at construction unless given.
+    """
+
+    def __init__(self, opt: dict, M: int, numels, stream: int | None = None):
+        import torch
+        if stream is None:
+            stream = torch.cuda.current_stream().cuda_stream
+        self.cfg = make_config(opt)
+        self.M = int(M)
+        self.h = mtdao_create(self.cfg, self.M, list(numels), stream)
+        lay = mtdao_layout(self.h)
+        self.n_padded = lay["n_padded"]
+        self.n_states = lay["n_states"]
+        self.offsets = lay["offsets"]
+        self.n_mom = int(opt["n_mom"])
+
+    def close(self) -> None:
+        if getattr(self, "h", None) is not None and self.h.value:
+            mtdao_destroy(self.h)
+            self.h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    @staticmethod
+    def _ptr(t) -> int:
+        return t if isinstance(t, int) else int(t.data_ptr())
+
+    def set_params(self, x0) -> None:
+        mtdao_set_params(self.h, self._ptr(x0))
+
+    def step(self, grads, lr: float, sync_mask: int | None = None, dtype: int | None = None) -> int:
+        """One local step; by default averages whatever is due at its end.
+        Returns the sync mask that was applied."""
+        if sync_mask is None:
+            sync_mask = mtdao_sync_due(self.h)
+        if dtype is None:
+            import torch
+            dtype = BF16 if grads.dtype == torch.bfloat16 else F32
+        mtdao_step(self.h, self._ptr(grads), dtype, lr, sync_mask)
+        return sync_mask
+
+    def step_host(self, grads_host, lr: float, sync_mask: int | None = None,
+                  dtype: int | None = None) -> int:
+        if sync_mask is None:
+            sync_mask = mtdao_sync_due(self.h)
+        if dtype is None:
+            import torch
+            dtype = BF16 if grads_host.dtype == torch.bfloat16 else F32
+        mtdao_step_host(self.h, self._ptr(grads_host), dtype, lr, sync_mask)
+        return sync_mask
+
+    def sync(self, mask: int) -> None:
+        mtdao_sync(self.h, mask)
+
+    def sync_due(self) -> int:
+        return mtdao_sync_due(self.h)
+
+    def state_ptr(self, state: int, replica: int) -> int:
+        return mtdao_get_state_ptr(self.h, state, replica)
+
+    def state_view(self, state: int):
+        """Torch view [M][n_padded] (fp32, device) of one state across replicas."""
+        import torch
+        ptr = mtdao_get_state_ptr(self.h, state, 0)
+        return _DevView.wrap(ptr, (self.M, self.n_padded))
+
+    @property
+    def t(self) -> int:
+        return mtdao_get_step(self.h)
+
+    @t.setter
+    def t(self, value: int) -> None:
+        mtdao_set_step(self.h, value)
+
+
+class _DevView:
+    """Zero-copy torch tensor over library-owned device memory (float32)."""
+
+    @staticmethod
+    def wrap(ptr: int, shape):
+        import torch
+
+        class _Cai:
+            def __init__(self, p, shp):
+                self.__cuda_array_interface__ = {
+                    "shape": tuple(shp), "typestr": "<f4", "data": (p, False), "version": 3,
+                    "strides": None}
+        return torch.as_tensor(_Cai(ptr, shape), device="cuda")

@@ -1,0 +1,76 @@
+// mtdao_internal.h -- shared between the C-ABI host code and the kernels.
+//
+// The per-step scalars are computed on the host in double precision from the
+// configuration and the step counter, rounded once to fp32 and passed to the
+// kernels by value (they live in the kernel parameter bank, not in memory).
+#pragma once
+
+#include <cuda_runtime.h>
+#include <cstdint>
+
+#include "mtdao.h"
+
+namespace mtdao {
+
+constexpr int kThreads = 256;        // threads per block of every streaming kernel
+constexpr int kChunk = 256;          // elements per warp iteration of the local step
+constexpr int kSyncChunk = 128;      // elements per warp iteration of the fused step+sync
+constexpr int kNormThreads = 256;    // threads per block of the norm reduction
+
+// Scalars of one local step t (Algorithms 1-3).  EMAs are evaluated as
+// s + c * (target - s) with c = 1 - beta, which keeps beta's precision when
+// beta is close to 1 (the float nearest 0.9999 is 1.7e-8 away from it, the
+// float nearest 1e-4 only 2.5e-12).
+struct StepScalars {
+    float neg_lr;                    // -eta_t
+    float c1[MTDAO_MAX_MOM];         // 1 - beta_{1,j}
+    float k[MTDAO_MAX_MOM];          // weight of u^j in Delta: omega_j / b_j (Adam), omega_j
+    float cg;                        // weight of the gradient term: 1 - sum omega
+    float c2;                        // 1 - beta_2
+    float sv;                        // Adam: 1 / sqrt(1 - beta_2^(t+1)), or 1
+    float eps;                       // epsilon
+    float clip_c;                    // ADOPT clamp bound c_t (+inf when not clipping)
+};
+
+struct StepArgs {
+    float *arena;                    // state-major arena, see mtdao.h "Layout"
+    const void *grads;               // [M][n_padded] f32 or bf16
+    const float *clip_scale;         // [M] global-norm clip factors, or nullptr
+    int64_t n_padded;                // elements per replica (multiple of 256)
+    int64_t stride;                  // M * n_padded: distance between two states
+    int32_t M;
+    uint32_t sync_mask;              // fused step+sync only
+    StepScalars sc;
+};
+
+struct SyncArgs {
+    float *arena;
+    int64_t n_padded;
+    int64_t stride;
+    int32_t M;
+    int32_t n_sel;                   // number of states to average
+    int32_t sel[2 + MTDAO_MAX_MOM];  // their indices
+};
+
+// Local step over all replicas (one pass).  Returns the launch error.
+cudaError_t launch_step(int base, int n_mom, int grad_dtype, bool clip, const StepArgs &a,
+                        int num_sms, cudaStream_t stream);
+
+// Local step with the replica average of the states in a.sync_mask fused
+// into the same pass.  Only for M in {2, 4, 8}; returns cudaErrorNotSupported
+// otherwise (the caller then runs launch_step followed by launch_sync).
+cudaError_t launch_step_sync(int base, int n_mom, int grad_dtype, bool clip, const StepArgs &a,
+                             int num_sms, cudaStream_t stream);
+
+// Replace each selected state by its mean over the M replicas.
+cudaError_t launch_sync(const SyncArgs &a, int num_sms, cudaStream_t stream);
+
+// Per-replica sum of squares of the gradient: partial sums into
+// partial[M][blocks_per_replica], then out[m] (double) and, when
+// clip_scale != nullptr, clip_scale[m] = min(1, rho / (sqrt(out[m]) + 1e-6)).
+int norm_blocks_per_replica(int num_sms, int M);
+cudaError_t launch_grad_sqnorm(const void *grads, int grad_dtype, int32_t M, int64_t n_padded,
+                               int blocks_per_replica, double *partial, double *out,
+                               float *clip_scale, double rho, cudaStream_t stream);
+
+}  // namespace mtdao

@@ -1,0 +1,160 @@
+// reduce_kernels.cu -- replica averaging (outer synchronisation) and the
+// per-replica gradient norm used by clip(g, rho).
+//
+// Averaging (Algorithms 1-3, E_m[.] with averaging as OuterOpt): for every
+// selected state and element, the M replica values are read once and the
+// mean is written back to all M replicas.  Algorithmic traffic: 8 * M bytes
+// per element per state.  HBM-bound; grid-stride over float4 vectors, one
+// grid row (blockIdx.y) per selected state.
+//
+// Norm: sum_i g[m][i]^2 per replica with a fixed grid and fixed reduction
+// order, so the result is bit-reproducible.  Each thread accumulates its
+// strided share in fp32 with Kahan compensation, warps and blocks combine in
+// fp64, and a second small kernel adds the per-block partials in order.
+#include <cuda_runtime.h>
+#include <cmath>
+#include <cstdint>
+
+#include "mtdao_internal.h"
+#include "step_kernels.cuh"
+
+namespace mtdao {
+
+namespace {
+
+template <int MT>
+__global__ void __launch_bounds__(kThreads) sync_kernel(const SyncArgs a) {
+    const int M = MT > 0 ? MT : a.M;
+    float *base = a.arena + static_cast<int64_t>(a.sel[blockIdx.y]) * a.stride;
+    const int64_t n = a.n_padded;
+    const int64_t nv = n / 4;
+    const float Mf = static_cast<float>(M);
+    for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < nv;
+         i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+        const int64_t e = 4 * i;
+        float s0[4], d[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+        to_array(ld_state(base + e), s0);
+        if constexpr (MT > 0) {
+            float r[MT][4];
+#pragma unroll
+            for (int m = 1; m < MT; ++m) to_array(ld_state(base + m * n + e), r[m]);
+#pragma unroll
+            for (int m = 1; m < MT; ++m)
+#pragma unroll
+                for (int k = 0; k < 4; ++k) d[k] += r[m][k] - s0[k];
+        } else {
+            for (int m = 1; m < M; ++m) {
+                float r[4];
+                to_array(ld_state(base + m * n + e), r);
+#pragma unroll
+                for (int k = 0; k < 4; ++k) d[k] += r[k] - s0[k];
+            }
+        }
+        float mean[4];
+#pragma unroll
+        for (int k = 0; k < 4; ++k) mean[k] = s0[k] + d[k] / Mf;
+        const float4 mv = from_array(mean);
+        for (int m = 0; m < M; ++m) st_state(base + m * n + e, mv);
+    }
+}
+
+template <int MT>
+cudaError_t launch_sync_t(const SyncArgs &a, int num_sms, cudaStream_t stream) {
+    static const int per_sm = blocks_per_sm(sync_kernel<MT>);
+    const int64_t nv = a.n_padded / 4;
+    int64_t gx = static_cast<int64_t>(per_sm) * num_sms / (a.n_sel > 0 ? a.n_sel : 1);
+    const int64_t need = (nv + kThreads - 1) / kThreads;
+    if (gx > need) gx = need;
+    if (gx < 1) gx = 1;
+    dim3 grid(static_cast<unsigned>(gx), static_cast<unsigned>(a.n_sel));
+    sync_kernel<MT><<<grid, kThreads, 0, stream>>>(a);
+    return cudaGetLastError();
+}
+
+__device__ __forceinline__ double warp_sum(double v) {
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) v += __shfl_down_sync(0xffffffffu, v, off);
+    return v;
+}
+
+// Deterministic block sum of one double per thread; result valid in thread 0.
+__device__ double block_sum(double v) {
+    __shared__ double part[kNormThreads / 32];
+    v = warp_sum(v);
+    const int w = threadIdx.x >> 5, l = threadIdx.x & 31;
+    if (l == 0) part[w] = v;
+    __syncthreads();
+    double total = 0.0;
+    if (threadIdx.x == 0)
+        for (int i = 0; i < static_cast<int>(blockDim.x >> 5); ++i) total += part[i];
+    return total;
+}
+
+template <int GDT>
+__global__ void __launch_bounds__(kNormThreads) sqnorm_partial_kernel(const void *g, int64_t n,
+                                                                      double *partial) {
+    const int m = blockIdx.y;
+    const int nb = gridDim.x;
+    const int64_t nv = n / 4;
+    float sum = 0.0f, comp = 0.0f;
+    for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < nv;
+         i += static_cast<int64_t>(nb) * blockDim.x) {
+        const float4 q = ld_grad<GDT>(g, m * n + 4 * i);
+        const float y = fmaf(q.x, q.x, fmaf(q.y, q.y, fmaf(q.z, q.z, __fmul_rn(q.w, q.w)))) - comp;
+        const float t = sum + y;
+        comp = (t - sum) - y;
+        sum = t;
+    }
+    const double total = block_sum(static_cast<double>(sum) - static_cast<double>(comp));
+    if (threadIdx.x == 0) partial[static_cast<int64_t>(m) * nb + blockIdx.x] = total;
+}
+
+__global__ void __launch_bounds__(kNormThreads) sqnorm_finalize_kernel(const double *partial, int nb,
+                                                                       double *out, float *clip_scale,
+                                                                       double rho) {
+    const int m = blockIdx.x;
+    double acc = 0.0;
+    for (int i = threadIdx.x; i < nb; i += blockDim.x) acc += partial[static_cast<int64_t>(m) * nb + i];
+    const double total = block_sum(acc);
+    if (threadIdx.x == 0) {
+        out[m] = total;
+        if (clip_scale != nullptr) {
+            const double f = rho / (sqrt(total) + 1e-6);
+            clip_scale[m] = static_cast<float>(f < 1.0 ? f : 1.0);
+        }
+    }
+}
+
+}  // namespace
+
+cudaError_t launch_sync(const SyncArgs &a, int num_sms, cudaStream_t stream) {
+    if (a.n_sel <= 0 || a.M <= 1) return cudaSuccess;
+    switch (a.M) {
+        case 2: return launch_sync_t<2>(a, num_sms, stream);
+        case 4: return launch_sync_t<4>(a, num_sms, stream);
+        case 8: return launch_sync_t<8>(a, num_sms, stream);
+        default: return launch_sync_t<0>(a, num_sms, stream);
+    }
+}
+
+int norm_blocks_per_replica(int num_sms, int M) {
+    int b = (4 * num_sms) / (M > 0 ? M : 1);
+    return b < 1 ? 1 : b;
+}
+
+cudaError_t launch_grad_sqnorm(const void *grads, int grad_dtype, int32_t M, int64_t n_padded,
+                               int blocks_per_replica, double *partial, double *out,
+                               float *clip_scale, double rho, cudaStream_t stream) {
+    dim3 grid(static_cast<unsigned>(blocks_per_replica), static_cast<unsigned>(M));
+    if (grad_dtype == MTDAO_F32)
+        sqnorm_partial_kernel<MTDAO_F32><<<grid, kNormThreads, 0, stream>>>(grads, n_padded, partial);
+    else
+        sqnorm_partial_kernel<MTDAO_BF16><<<grid, kNormThreads, 0, stream>>>(grads, n_padded, partial);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    sqnorm_finalize_kernel<<<M, kNormThreads, 0, stream>>>(partial, blocks_per_replica, out, clip_scale,
+                                                          rho);
+    return cudaGetLastError();
+}
+
+}  // namespace mtdao

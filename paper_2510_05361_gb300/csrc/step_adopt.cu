@@ -1,0 +1,12 @@
+// step_adopt.cu -- instantiates the local-step kernels of Algorithm 2 (MT-DAO-ADOPT).
+// One translation unit per base so that the instantiations compile in parallel.
+#include "step_kernels.cuh"
+
+namespace mtdao {
+
+template cudaError_t launch_step_base<MTDAO_BASE_ADOPT>(int, int, bool, const StepArgs &, int,
+                                                cudaStream_t);
+template cudaError_t launch_step_sync_base<MTDAO_BASE_ADOPT>(int, int, bool, const StepArgs &, int,
+                                                     cudaStream_t);
+
+}  // namespace mtdao

@@ -16,8 +16,8 @@ Hyper-parameters the paper leaves open are chosen as follows:
 
 Layout convention (shared with the library, which computes it on its own):
 each tensor starts at a multiple of 8 elements (32 B of fp32, 16 B of bf16)
-and the per-worker length ``n_padded`` is rounded up to a multiple of 64
-elements (256 B) so every worker's slab starts 256-byte aligned.
+and the per-worker length ``n_padded`` is rounded up to a multiple of 256
+elements (1 KiB) so every worker's slab starts 1024-byte aligned.
 """
 from __future__ import annotations
 
@@ -27,7 +27,7 @@ VOCAB = 50257
 INIT_SEED = 20251005
 GRAD_SEED = INIT_SEED + 1
 TENSOR_ALIGN = 8
-SLAB_ALIGN = 64
+SLAB_ALIGN = 256
 
 
 def decoder_shapes(vocab: int, d: int, ffn: int, blocks: int) -> list[int]:

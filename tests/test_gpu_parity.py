@@ -1,0 +1,315 @@
+"""GPU parity: the CUDA library (through its C ABI) against the CPU oracle.
+
+Every case runs the library's kernels on seeded inputs and the oracle on the
+same inputs (host generator), then compares every state of every replica
+with the tolerance of ``parity_util`` (1e-5 relative, RMS floor).
+"""
+import ctypes
+
+import numpy as np
+import pytest
+
+torch = pytest.importorskip("torch")
+
+from parity_util import (TOL, compare, host_grads, oracle_run, rel_err, sample_indices,
+                         state_names, workload_dict)
+from synth import generators as G
+from synth import workloads as W
+
+pytestmark = pytest.mark.gpu
+
+SEED_G, SEED_I = 1234, 5678
+
+
+@pytest.fixture(scope="module")
+def P():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    import paper_2510_05361_gb300 as P
+    P.load()
+    return P
+
+
+def to_dev(g_np, gdt):
+    t = torch.from_numpy(np.ascontiguousarray(g_np)).cuda()
+    return t.to(torch.bfloat16) if gdt == "bf16" else t
+
+
+def gpu_run(P, w, T, fused=True, lr=None, t0=0, eng=None, x0=None):
+    lay = W.layout(w["shapes"])
+    n = lay["n_padded"]
+    opt = w["opt"]
+    lr = opt.get("lr", 1e-3) if lr is None else lr
+    idx = np.arange(n)
+    if eng is None:
+        eng = P.MTDAO(opt, w["M"], w["shapes"])
+        if x0 is None:
+            x0 = G.init_params(w, lay, SEED_I, idx)
+        eng.set_params(torch.from_numpy(x0).cuda())
+    for t in range(t0, t0 + T):
+        g = to_dev(host_grads(w, lay, SEED_G, t, idx), w["grad_dtype"])
+        due = eng.sync_due()
+        if fused:
+            eng.step(g, lr, due)
+        else:
+            eng.step(g, lr, 0)
+            eng.sync(due)
+    torch.cuda.synchronize()
+    return eng
+
+
+def gpu_states(eng, opt):
+    out = {}
+    for s, name in enumerate(state_names(opt)):
+        out[name] = eng.state_view(s).cpu().numpy()
+    return out
+
+
+RAGGED = [1, 7, 300, 4099, 2560, 13]
+
+
+@pytest.mark.parametrize("gdt", ["f32", "bf16"])
+@pytest.mark.parametrize("N", [1, 2, 3, 4])
+@pytest.mark.parametrize("base", ["adam", "adopt", "sgdm"])
+@pytest.mark.parametrize("M", [3, 4])
+def test_step_and_sync_parity_matrix(P, base, N, gdt, M):
+    betas = W.SWEEP_BETAS[:N]
+    w = workload_dict(RAGGED, M, base=base, betas=betas, beta2=0.9999 if base == "adopt" else 0.999,
+                      px=5, pu=[3, 4, 2, 6][:N], pv=4, lr=2.0 ** -8 if base == "adopt" else 1e-3,
+                      gdt=gdt)
+    T = 13
+    eng = gpu_run(P, w, T)
+    lay = W.layout(w["shapes"])
+    ref = oracle_run(w["opt"], M, np.arange(lay["n_padded"]), T, lay, w, SEED_G, SEED_I)
+    compare(gpu_states(eng, w["opt"]), ref)
+    eng.close()
+
+
+@pytest.mark.parametrize("M", [1, 2, 5, 8])
+def test_replica_counts(P, M):
+    w = workload_dict([5000, 123], M, betas=(0.9, 0.999), px=4, pu=2, pv=3)
+    eng = gpu_run(P, w, 9)
+    lay = W.layout(w["shapes"])
+    ref = oracle_run(w["opt"], M, np.arange(lay["n_padded"]), 9, lay, w, SEED_G, SEED_I)
+    compare(gpu_states(eng, w["opt"]), ref)
+    eng.close()
+
+
+def test_fused_sync_is_bitwise_equal_to_separate_sync(P):
+    for base, M in (("adam", 4), ("adopt", 8), ("sgdm", 2)):
+        w = workload_dict(RAGGED, M, base=base, betas=(0.9, 0.99, 0.5), px=3, pu=[2, 3, 4], pv=2,
+                          beta2=0.9999 if base == "adopt" else 0.999)
+        a = gpu_run(P, w, 8, fused=True)
+        b = gpu_run(P, w, 8, fused=False)
+        sa, sb = gpu_states(a, w["opt"]), gpu_states(b, w["opt"])
+        for k in sa:
+            assert np.array_equal(sa[k].view(np.uint32), sb[k].view(np.uint32)), (base, k)
+        a.close()
+        b.close()
+
+
+@pytest.mark.parametrize("base", ["adam", "sgdm"])
+def test_global_norm_clip_parity(P, base):
+    # sigma = 1 gives ||g|| ~ 90 >> rho = 1: clipping is active every step
+    w = workload_dict([5000, 3001, 17], 4, base=base, betas=(0.9, 0.999), clip="global_norm",
+                      rho=1.0, px=3, pu=2, pv=3, sigma=1.0)
+    eng = gpu_run(P, w, 10)
+    lay = W.layout(w["shapes"])
+    ref = oracle_run(w["opt"], 4, np.arange(lay["n_padded"]), 10, lay, w, SEED_G, SEED_I)
+    compare(gpu_states(eng, w["opt"]), ref)
+    eng.close()
+
+
+@pytest.mark.parametrize("gdt", ["f32", "bf16"])
+def test_grad_sqnorm(P, gdt):
+    w = workload_dict([70000, 3, 1000], 3, sigma=0.5, gdt=gdt)
+    lay = W.layout(w["shapes"])
+    g = host_grads(w, lay, SEED_G, 0, np.arange(lay["n_padded"]))
+    eng = P.MTDAO(w["opt"], 3, w["shapes"])
+    out = torch.zeros(3, dtype=torch.float64, device="cuda")
+    gd = to_dev(g, gdt)
+    P.mtdao_grad_sqnorm(eng.h, gd.data_ptr(), P.BF16 if gdt == "bf16" else P.F32, out.data_ptr())
+    got = out.cpu().numpy()
+    expect = np.sum(g.astype(np.float64) ** 2, axis=1)
+    assert np.max(np.abs(got - expect) / expect) < 1e-6
+    again = torch.zeros_like(out)
+    P.mtdao_grad_sqnorm(eng.h, gd.data_ptr(), P.BF16 if gdt == "bf16" else P.F32, again.data_ptr())
+    assert torch.equal(out, again)           # deterministic
+    eng.close()
+
+
+@pytest.mark.parametrize("clip", ["elementwise", "none"])
+def test_adopt_clip_parity(P, clip):
+    w = workload_dict(RAGGED, 4, base="adopt", betas=(0.95, 0.999), beta2=0.9999, clip=clip,
+                      px=6, pu=3, pv=3, lr=2.0 ** -8)
+    eng = gpu_run(P, w, 20)
+    lay = W.layout(w["shapes"])
+    ref = oracle_run(w["opt"], 4, np.arange(lay["n_padded"]), 20, lay, w, SEED_G, SEED_I)
+    compare(gpu_states(eng, w["opt"]), ref)
+    eng.close()
+
+
+def test_alg2_literal_phase_parity(P):
+    w = workload_dict(RAGGED, 4, base="adopt", betas=(0.95,), beta2=0.9999, px=4, pu=3, pv=5,
+                      phase="alg2_literal", lr=2.0 ** -8)
+    eng = gpu_run(P, w, 14)
+    lay = W.layout(w["shapes"])
+    ref = oracle_run(w["opt"], 4, np.arange(lay["n_padded"]), 14, lay, w, SEED_G, SEED_I)
+    compare(gpu_states(eng, w["opt"]), ref)
+    eng.close()
+
+
+def test_sync_kernel_parity_and_invariants(P):
+    M, shapes = 4, [20000, 11]
+    w = workload_dict(shapes, M, betas=(0.9, 0.99))
+    eng = P.MTDAO(w["opt"], M, shapes)
+    n = eng.n_padded
+    rng = np.random.default_rng(3)
+    vals = {}
+    for s in range(eng.n_states):
+        arr = rng.standard_normal((M, n)).astype(np.float32)
+        if s == eng.n_states - 1:
+            arr = np.abs(arr)
+        vals[s] = arr
+        eng.state_view(s).copy_(torch.from_numpy(arr).cuda())
+    eng.sync(0b1011)                       # x, u1, v
+    torch.cuda.synchronize()
+    for s in range(eng.n_states):
+        got = eng.state_view(s).cpu().numpy()
+        if (0b1011 >> s) & 1:
+            expect = np.broadcast_to(vals[s].astype(np.float64).mean(0), (M, n))
+            assert rel_err(got, expect) <= 2 * np.finfo(np.float32).eps
+            assert np.all(got == got[0:1])
+        else:
+            assert np.array_equal(got, vals[s])
+    before = {s: eng.state_view(s).cpu().numpy().copy() for s in range(eng.n_states)}
+    eng.sync(0b1011)                       # idempotent: replicas now agree
+    torch.cuda.synchronize()
+    for s in range(eng.n_states):
+        assert np.array_equal(eng.state_view(s).cpu().numpy(), before[s])
+    eng.close()
+
+
+@pytest.mark.parametrize("M", [1, 3, 4, 6, 8])
+def test_sync_identity_on_identical_replicas(P, M):
+    w = workload_dict([777, 4096], M, betas=(0.9,))
+    eng = P.MTDAO(w["opt"], M, w["shapes"])
+    rng = np.random.default_rng(M)
+    for s in range(eng.n_states):
+        row = rng.standard_normal(eng.n_padded).astype(np.float32)
+        eng.state_view(s).copy_(torch.from_numpy(np.tile(row, (M, 1))).cuda())
+    before = {s: eng.state_view(s).cpu().numpy().copy() for s in range(eng.n_states)}
+    eng.sync((1 << eng.n_states) - 1)
+    torch.cuda.synchronize()
+    for s in range(eng.n_states):
+        assert np.array_equal(eng.state_view(s).cpu().numpy().view(np.uint32),
+                              before[s].view(np.uint32))
+    eng.close()
+
+
+def test_host_gradient_path_is_bitwise_equal(P):
+    w = workload_dict(RAGGED, 4, betas=(0.9, 0.999), px=3, pu=3, pv=3)
+    lay = W.layout(w["shapes"])
+    idx = np.arange(lay["n_padded"])
+    a = gpu_run(P, w, 7)
+    b = P.MTDAO(w["opt"], 4, w["shapes"])
+    b.set_params(torch.from_numpy(G.init_params(w, lay, SEED_I, idx)).cuda())
+    for t in range(7):
+        g = torch.from_numpy(host_grads(w, lay, SEED_G, t, idx)).pin_memory()
+        b.step_host(g, 1e-3)
+        torch.cuda.current_stream().synchronize()
+    sa, sb = gpu_states(a, w["opt"]), gpu_states(b, w["opt"])
+    for k in sa:
+        assert np.array_equal(sa[k], sb[k]), k
+    a.close()
+    b.close()
+
+
+def test_checkpoint_resume_is_bitwise_equal(P):
+    w = workload_dict(RAGGED, 4, betas=(0.9, 0.999), px=4, pu=3, pv=4)
+    full = gpu_run(P, w, 10)
+    first = gpu_run(P, w, 6)
+    saved = {s: first.state_view(s).cpu().numpy().copy() for s in range(first.n_states)}
+    step = first.t
+    first.close()
+    resumed = P.MTDAO(w["opt"], 4, w["shapes"])
+    for s, arr in saved.items():
+        for m in range(4):
+            row = np.ascontiguousarray(arr[m])
+            P.mtdao_copy_state_from_host(resumed.h, s, m, row.ctypes.data)
+    resumed.t = step
+    gpu_run(P, w, 4, t0=6, eng=resumed)
+    sf, sr = gpu_states(full, w["opt"]), gpu_states(resumed, w["opt"])
+    for k in sf:
+        assert np.array_equal(sf[k], sr[k]), k
+    full.close()
+    resumed.close()
+
+
+def test_nonfinite_gradients_propagate_like_the_oracle(P):
+    w = workload_dict([1000], 2, betas=(0.9,), px=0, pu=0, pv=0)
+    lay = W.layout(w["shapes"])
+    idx = np.arange(lay["n_padded"])
+    eng = P.MTDAO(w["opt"], 2, w["shapes"])
+    x0 = G.init_params(w, lay, SEED_I, idx)
+    eng.set_params(torch.from_numpy(x0).cuda())
+    g = host_grads(w, lay, SEED_G, 0, idx)
+    g[0, 5] = np.nan
+    g[1, 9] = np.inf
+    eng.step(torch.from_numpy(g).cuda(), 1e-3, 0)
+    torch.cuda.synchronize()
+    from oracle.oracle import Oracle
+    o = Oracle(w["opt"], 2, lay["n_padded"], x0=x0.astype(np.float64))
+    o.step(0, 1e-3, g.astype(np.float64))
+    compare(gpu_states(eng, w["opt"]), o.states())
+    eng.close()
+
+
+def test_error_codes(P, monkeypatch):
+    w = workload_dict([1024], 2, betas=(0.9,))
+    eng = P.MTDAO(w["opt"], 2, w["shapes"])
+    g = torch.zeros(2 * eng.n_padded + 4, device="cuda")
+    with pytest.raises(P.MTDAOError) as e:
+        P.mtdao_step(eng.h, g.data_ptr() + 4, P.F32, 1e-3, 0)
+    assert e.value.code == P.ERR_ALIGN
+    with pytest.raises(P.MTDAOError) as e:
+        P.mtdao_step(eng.h, g.data_ptr(), 7, 1e-3, 0)
+    assert e.value.code == P.ERR_INVALID
+    with pytest.raises(P.MTDAOError) as e:
+        P.mtdao_step(eng.h, g.data_ptr(), P.F32, 1e-3, 1 << eng.n_states)
+    assert e.value.code == P.ERR_INVALID
+    with pytest.raises(P.MTDAOError) as e:
+        P.mtdao_sync(eng.h, 1 << 5)
+    assert e.value.code == P.ERR_INVALID
+    assert eng.t == 0
+    eng.close()
+    free0 = torch.cuda.mem_get_info()[0]
+    for k in (1, 2, 3, 4):
+        monkeypatch.setenv("MTDAO_FAULT_ALLOC", str(k))
+        with pytest.raises(P.MTDAOError) as e:
+            P.mtdao_create(P.make_config(w["opt"]), 2, [1 << 20])
+        assert e.value.code == P.ERR_OOM
+        assert "failed" in P.mtdao_last_error(None)
+    monkeypatch.delenv("MTDAO_FAULT_ALLOC")
+    torch.cuda.synchronize()
+    assert abs(torch.cuda.mem_get_info()[0] - free0) < (64 << 20)
+
+
+def test_device_generator_matches_host_generator(P):
+    from synth.device import DeviceInputs
+    for name in ("tiny", "gpt2_small", "decoder_350m", "decoder_1b"):
+        w = W.get(name)
+        w["M"] = min(w["M"], 2)
+        w["shapes"] = w["shapes"][:3] + [1001]
+        lay = W.layout(w["shapes"])
+        dev = DeviceInputs(w, lay, SEED_G, SEED_I)
+        idx = sample_indices(lay, 5000, seed=1)
+        for t in (0, 7):
+            got = dev.grads(t)
+            if w["grad_dtype"] == "bf16":
+                got = got.float()
+            got = got.cpu().numpy()[:, idx]
+            expect = host_grads(w, lay, SEED_G, t, idx)
+            assert np.array_equal(got.view(np.uint32), expect.view(np.uint32)), name
+        x0 = dev.init_params().cpu().numpy()[idx]
+        assert np.array_equal(x0, G.init_params(w, lay, SEED_I, idx))
