@@ -123,6 +123,20 @@ WORKLOADS = {
         "init_sigma": 0.02,
         "opt": _opt("adam", (0.5, 0.9, 0.999), 0.999, 1e-3, 32, 32, 32),
     },
+    "profile_small": {
+        "name": "profile_small",
+        "desc": "flat fp32 vector n=2^25 with the ~1B workload's optimizer (M=4, N=3 "
+                "beta=(0.5,0.9,0.999), Adam, grads N(0,1e-3) with 1% outliers x100, H=32): "
+                "the same kernels on ~3 GB of device memory, for profiler captures",
+        "shapes": [1 << 25],
+        "M": 4,
+        "T": 64,
+        "grad_kind": "normal_outliers",
+        "grad_sigma": 1e-3,
+        "grad_dtype": "f32",
+        "init_sigma": 0.02,
+        "opt": _opt("adam", (0.5, 0.9, 0.999), 0.999, 1e-3, 32, 32, 32),
+    },
 }
 
 SWEEP_BETAS = (0.9, 0.999, 0.5, 0.99)
