@@ -231,6 +231,44 @@ int mtdao_sync_due(mtdao_handle h, uint32_t *mask_out);
 int mtdao_grad_sqnorm(mtdao_handle h, const void *grads_dev, int32_t grad_dtype,
                       double *out_dev);
 
+/*
+ * mtdao_grad_sqnorm_static -- the per-replica sum of squares of
+ * mtdao_grad_sqnorm for callers that cannot allocate device memory.
+ * The paper has no counterpart; this is a library convenience.
+ *
+ * Who needs it: a process whose device memory is reserved up front by
+ * another allocator (so a cudaMalloc from this library would fail), a
+ * latency-critical loop in which cudaMalloc/cudaFree would synchronise the
+ * device, or a hook that sees only a gradient buffer and holds no handle
+ * (mtdao_create allocates).  This call allocates nothing: neither
+ * cudaMalloc/cudaFree nor any allocating library routine.
+ *
+ * Scratch: its per-block partial sums live in one file-scope device array
+ * of MTDAO_STATIC_SCRATCH_DOUBLES doubles (32 KiB), which every device that
+ * loads the library holds until the process exits.  A call needs
+ * M * blocks_per_replica slots (blocks_per_replica = max(1, 4 * SMs / M),
+ * the grid of mtdao_grad_sqnorm, so both return the same bits); a call that
+ * would need more fails with MTDAO_ERR_INVALID and a message.  Every slot a
+ * call reads is written earlier in the same call, so nothing has to be
+ * cleared between calls; the array keeps the last call's partial sums.
+ * All calls on a device share the array: calls whose GPU work overlaps (on
+ * different streams or from different threads) race and return garbage.
+ *
+ * Set-up: the first call on a device (with that device current) looks up
+ * the array's device address with cudaGetSymbolAddress and caches it; make
+ * that first call before any stream capture begins.
+ *
+ * grads_dev: device, [M][n_padded] of grad_dtype, 16-byte aligned;
+ * n_padded a positive multiple of 256; 1 <= M <= MTDAO_MAX_REPLICAS.
+ * out_dev: device, M doubles (caller-owned), receives sum_i g[m][i]^2.
+ * cuda_stream: cudaStream_t the work is enqueued on (asynchronous).
+ * Errors: MTDAO_ERR_INVALID, MTDAO_ERR_ALIGN, MTDAO_ERR_CUDA; the message is
+ * available from mtdao_last_error(NULL) in the calling thread.
+ */
+#define MTDAO_STATIC_SCRATCH_DOUBLES 4096
+int mtdao_grad_sqnorm_static(const void *grads_dev, int32_t grad_dtype, int32_t M,
+                             int64_t n_padded, double *out_dev, void *cuda_stream);
+
 /* ------------------------------------------------------------------ state access */
 
 /* Device pointer to state `state` of replica `replica` ([n_padded] fp32). */
@@ -259,7 +297,8 @@ int mtdao_set_step(mtdao_handle h, int64_t step);
 
 /*
  * Message of the handle's last failure ("" if none).  With h == NULL: the
- * last failure of mtdao_create / mtdao_config_validate in this thread.
+ * last failure of a call without a handle (mtdao_create,
+ * mtdao_config_validate, mtdao_grad_sqnorm_static, ...) in this thread.
  */
 const char *mtdao_last_error(mtdao_handle h);
 

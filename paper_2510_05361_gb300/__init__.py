@@ -83,6 +83,8 @@ def _load():
         "mtdao_sync": (ctypes.c_int, [H, ctypes.c_uint32]),
         "mtdao_sync_due": (ctypes.c_int, [H, ctypes.POINTER(ctypes.c_uint32)]),
         "mtdao_grad_sqnorm": (ctypes.c_int, [H, ctypes.c_void_p, ctypes.c_int32, ctypes.c_void_p]),
+        "mtdao_grad_sqnorm_static": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_int32, ctypes.c_int32,
+                                                    ctypes.c_int64, ctypes.c_void_p, ctypes.c_void_p]),
         "mtdao_get_state_ptr": (ctypes.c_int, [H, ctypes.c_int32, ctypes.c_int32,
                                                ctypes.POINTER(ctypes.c_void_p)]),
         "mtdao_copy_state_to_host": (ctypes.c_int, [H, ctypes.c_int32, ctypes.c_int32, ctypes.c_void_p]),
@@ -225,6 +227,13 @@ def mtdao_sync_due(h) -> int:
 def mtdao_grad_sqnorm(h, grads_dev_ptr: int, grad_dtype: int, out_dev_ptr: int) -> None:
     _check(lib.mtdao_grad_sqnorm(h, ctypes.c_void_p(grads_dev_ptr), grad_dtype,
                                  ctypes.c_void_p(out_dev_ptr)), h)
+
+
+def mtdao_grad_sqnorm_static(grads_dev_ptr: int, grad_dtype: int, M: int, n_padded: int,
+                             out_dev_ptr: int, stream: int = 0) -> None:
+    """Allocation-free per-replica sum of squares (no handle needed)."""
+    _check(lib.mtdao_grad_sqnorm_static(ctypes.c_void_p(grads_dev_ptr), grad_dtype, M, n_padded,
+                                        ctypes.c_void_p(out_dev_ptr), ctypes.c_void_p(stream)))
 
 
 def mtdao_get_state_ptr(h, state: int, replica: int) -> int:

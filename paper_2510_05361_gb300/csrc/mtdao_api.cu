@@ -256,6 +256,8 @@ int select_device(mtdao_ctx *h) {
 
 }  // namespace
 
+int mtdao::set_thread_error(int code, const char *msg) { return set_error(nullptr, code, "%s", msg); }
+
 // ====================================================================== host-only
 
 extern "C" int32_t mtdao_version(void) { return MTDAO_VERSION; }

@@ -73,4 +73,8 @@ cudaError_t launch_grad_sqnorm(const void *grads, int grad_dtype, int32_t M, int
                                int blocks_per_replica, double *partial, double *out,
                                float *clip_scale, double rho, cudaStream_t stream);
 
+// Record a message for mtdao_last_error(NULL) in the calling thread and
+// return code (for entry points that have no handle).
+int set_thread_error(int code, const char *msg);
+
 }  // namespace mtdao
