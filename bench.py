@@ -36,7 +36,7 @@ if ROOT not in sys.path:
 from synth import workloads as W  # noqa: E402
 
 PEAKS_FILE = os.path.join(ROOT, "MEASURED_PEAKS.json")
-TRAFFIC_FILE = os.path.join(ROOT, "profiles", "step_kernel_traffic.json")
+TRAFFIC_FILE = os.path.join(ROOT, "profiles", "step_kernel_traffic.txt")
 STEP_KERNEL_SRC = os.path.join(ROOT, "paper_2510_05361_gb300", "csrc", "step_kernels.cuh")
 FALLBACK_HBM_GBS = 6800.0
 L2_BYTES = 129 * 2 ** 20
@@ -75,15 +75,21 @@ def source_sha() -> str:
 
 def measured_traffic(workload: str, per_launch_units: int):
     """DRAM bytes per launch of the step kernel from the committed ncu
-    summary, scaled to this launch; None if absent or the kernel changed."""
+    summary, scaled by elements to this launch; None if absent or if the
+    kernel source changed since the capture."""
+    rec = {}
     try:
         with open(TRAFFIC_FILE) as f:
-            rec = json.load(f)
+            for line in f:
+                line = line.strip()
+                if line and not line.startswith("#") and "=" in line:
+                    k, v = line.split("=", 1)
+                    rec[k] = v
+        if rec.get("source_sha") != source_sha():
+            return None
+        per_unit = float(rec["dram_bytes"]) / float(rec["elements"])
     except Exception:
         return None
-    if rec.get("source_sha") != source_sha():
-        return None
-    per_unit = rec["dram_bytes"] / rec["elements"]
     return int(round(per_unit * per_launch_units))
 
 

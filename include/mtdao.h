@@ -201,11 +201,13 @@ int mtdao_step(mtdao_handle h, const void *grads_dev, int32_t grad_dtype, double
                uint32_t sync_mask);
 
 /*
- * mtdao_step with the gradients in host memory: they are copied to a
- * library-owned device staging buffer (allocated on first use, two buffers
- * so that a copy can overlap the previous step) and the step runs from
- * there.  grads_host should be pinned for the copy to be asynchronous; it
- * must stay unchanged until the call's work on the stream has completed.
+ * mtdao_step with the gradients in host memory ([M][n_padded], 16-byte
+ * aligned).  Pinned memory (cudaHostAlloc / cudaHostRegister) is read by the
+ * step kernel directly over the host link, with no copy and no staging
+ * memory.  Other (pageable) memory is first copied into a library-owned
+ * device staging buffer (two buffers, allocated on first use, so that a
+ * copy can overlap the previous step).  grads_host must stay unchanged until
+ * the call's work on the stream has completed.
  */
 int mtdao_step_host(mtdao_handle h, const void *grads_host, int32_t grad_dtype, double lr,
                     uint32_t sync_mask);

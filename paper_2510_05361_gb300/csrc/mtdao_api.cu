@@ -489,6 +489,14 @@ extern "C" int mtdao_step_host(mtdao_handle h, const void *grads_host, int32_t g
     if (grad_dtype != MTDAO_F32 && grad_dtype != MTDAO_BF16)
         return set_error(h, MTDAO_ERR_INVALID, "unknown gradient dtype %d", grad_dtype);
     if (int rc = select_device(h)) return rc;
+    // Pinned (page-locked or registered) host memory is directly addressable
+    // by the GPU: the step kernel streams the gradients over the host link
+    // itself, with no staging copy and no staging memory.
+    cudaPointerAttributes attr;
+    if (cudaPointerGetAttributes(&attr, grads_host) == cudaSuccess && attr.type == cudaMemoryTypeHost &&
+        attr.devicePointer != nullptr)
+        return mtdao_step(h, attr.devicePointer, grad_dtype, lr, sync_mask);
+    cudaGetLastError();
     const size_t full = static_cast<size_t>(h->M) * h->n_padded * sizeof(float);
     const size_t bytes = static_cast<size_t>(h->M) * h->n_padded * (grad_dtype == MTDAO_BF16 ? 2 : 4);
     cudaError_t e;

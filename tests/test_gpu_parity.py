@@ -212,7 +212,10 @@ def test_sync_identity_on_identical_replicas(P, M):
     eng.close()
 
 
-def test_host_gradient_path_is_bitwise_equal(P):
+@pytest.mark.parametrize("memory", ["pinned", "pageable"])
+def test_host_gradient_path_is_bitwise_equal(P, memory):
+    """Pinned host gradients are read by the kernel over the host link;
+    pageable ones go through the staging copy.  Both equal the device path."""
     w = workload_dict(RAGGED, 4, betas=(0.9, 0.999), px=3, pu=3, pv=3)
     lay = W.layout(w["shapes"])
     idx = np.arange(lay["n_padded"])
@@ -220,8 +223,12 @@ def test_host_gradient_path_is_bitwise_equal(P):
     b = P.MTDAO(w["opt"], 4, w["shapes"])
     b.set_params(torch.from_numpy(G.init_params(w, lay, SEED_I, idx)).cuda())
     for t in range(7):
-        g = torch.from_numpy(host_grads(w, lay, SEED_G, t, idx)).pin_memory()
-        b.step_host(g, 1e-3)
+        g = np.ascontiguousarray(host_grads(w, lay, SEED_G, t, idx))
+        if memory == "pinned":
+            gt = torch.from_numpy(g).pin_memory()
+            b.step_host(gt, 1e-3)
+        else:
+            b.step_host(g.ctypes.data, 1e-3, dtype=P.F32)
         torch.cuda.current_stream().synchronize()
     sa, sb = gpu_states(a, w["opt"]), gpu_states(b, w["opt"])
     for k in sa:
