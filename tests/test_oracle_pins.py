@@ -277,6 +277,25 @@ def test_global_norm_clip():
     assert rel(a.v, (1 - 0.999) * g_big ** 2) < 1e-12
 
 
+def test_sgdm_constant_gradient_closed_form():
+    """Algorithm 3 under a constant gradient: u_j(t) = (1-beta_j^(t+1)) g, so
+    Delta_t = [(1 - sum w) + sum w_j (1-beta_j^(t+1))] g, unnormalised."""
+    betas, om = (0.5, 0.9, 0.99), (0.2, 0.3, 0.4)
+    c = cfg("sgdm", betas, omega=om)
+    rng = np.random.default_rng(15)
+    M, n, T = 2, 30, 25
+    g = rng.standard_normal((M, n))
+    x0 = rng.standard_normal(n)
+    o = Oracle(c, M, n, x0=x0)
+    x = np.broadcast_to(x0, (M, n)).copy()
+    for t in range(T):
+        lr = 0.01 * (1 + 0.1 * t)
+        o.step(t, lr, g)
+        w = (1 - sum(om)) + sum(o_ * (1 - b ** (t + 1)) for o_, b in zip(om, betas))
+        x = x - lr * w * g
+    assert np.max(np.abs(o.x - x)) < 1e-13
+
+
 # ------------------------------------------------------------ ADOPT pins
 
 @pytest.mark.parametrize("clip", ["elementwise", "none"])
