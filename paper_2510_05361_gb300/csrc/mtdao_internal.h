@@ -14,7 +14,6 @@ namespace mtdao {
 
 constexpr int kThreads = 256;        // threads per block of every streaming kernel
 constexpr int kChunk = 256;          // elements per warp iteration of the local step
-constexpr int kSyncChunk = 128;      // elements per warp iteration of the fused step+sync
 constexpr int kNormThreads = 256;    // threads per block of the norm reduction
 
 // Scalars of one local step t (Algorithms 1-3).  EMAs are evaluated as

@@ -1,6 +1,7 @@
 // step_adam.cu -- instantiates the local-step kernels of Algorithm 1 (MT-DAO-Adam).
 // One translation unit per base so that the instantiations compile in parallel.
 #include "step_kernels.cuh"
+#include "step_sync_kernels.cuh"
 
 namespace mtdao {
 

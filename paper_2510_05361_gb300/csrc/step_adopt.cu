@@ -1,6 +1,7 @@
 // step_adopt.cu -- instantiates the local-step kernels of Algorithm 2 (MT-DAO-ADOPT).
 // One translation unit per base so that the instantiations compile in parallel.
 #include "step_kernels.cuh"
+#include "step_sync_kernels.cuh"
 
 namespace mtdao {
 

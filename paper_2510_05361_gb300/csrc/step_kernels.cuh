@@ -1,4 +1,4 @@
-// step_kernels.cuh -- the fused MT-DAO local step (Algorithms 1-3) for sm_103a.
+// step_kernels.cuh -- the MT-DAO local step (Algorithms 1-3) for sm_103a.
 //
 // The step is elementwise and HBM-bound (about 0.3 flop per byte), so it is
 // written as a persistent grid-stride streaming kernel: every state of every
@@ -8,14 +8,10 @@
 // of the chunk, so every warp-wide load or store instruction covers 512
 // contiguous bytes of fp32 (256 bytes of bf16 gradient).
 //
-// Two kernels share one per-element update:
-//   step_kernel       replica-major: the flat index runs over all M replicas
-//                     (M * n_padded elements); used for steps with no sync.
-//   step_sync_kernel  element-major: a lane updates the same 4 elements of
-//                     all M replicas, then writes each state due for
-//                     averaging as the replica mean (Algorithm 1's E_m[.])
-//                     instead of the M local values.  The average costs no
-//                     HBM traffic beyond the step's own.
+// This header holds the per-element update shared by both step kernels and
+// step_kernel, which is replica-major: the flat index runs over all M
+// replicas (M * n_padded elements); it serves every step with no average.
+// The fused step + average kernel is in step_sync_kernels.cuh.
 #pragma once
 
 #include <cuda_runtime.h>
@@ -156,150 +152,6 @@ __global__ void __launch_bounds__(kThreads) step_kernel(const StepArgs a) {
     }
 }
 
-// ---------------------------------------------------------------- fused step + sync
-
-// Writes the M replicas' values of one state for 4 elements: either as they
-// are, or (when the state is due) all M replaced by the replica mean
-// s_0 + (sum_{m>=1} (s_m - s_0)) / M, summed in replica order.  The
-// standalone averaging kernel uses the same expression and order, so fused
-// and separate averaging give identical bits.
-template <int M>
-__device__ __forceinline__ void store_replicas(float *state, int64_t n_padded, int64_t e,
-                                               float (&val)[M][4], bool average) {
-    if (average) {
-        float mean[4];
-#pragma unroll
-        for (int k = 0; k < 4; ++k) {
-            float d = 0.0f;
-#pragma unroll
-            for (int m = 1; m < M; ++m) d += val[m][k] - val[0][k];
-            mean[k] = val[0][k] + d / static_cast<float>(M);
-        }
-#pragma unroll
-        for (int m = 0; m < M; ++m) st_state(state + m * n_padded + e, from_array(mean));
-    } else {
-#pragma unroll
-        for (int m = 0; m < M; ++m) st_state(state + m * n_padded + e, from_array(val[m]));
-    }
-}
-
-template <int M>
-__device__ __forceinline__ void load_replicas(const float *state, int64_t n_padded, int64_t e,
-                                              float (&val)[M][4]) {
-#pragma unroll
-    for (int m = 0; m < M; ++m) to_array(ld_state(state + m * n_padded + e), val[m]);
-}
-
-template <int BASE, int N, int GDT, bool CLIP, int M>
-__global__ void __launch_bounds__(kThreads) step_sync_kernel(const StepArgs a) {
-    const int lane = threadIdx.x & 31;
-    const int64_t n = a.n_padded;
-    const int64_t n_chunks = n / kSyncChunk;
-    const int64_t warp = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
-    const int64_t n_warps = (static_cast<int64_t>(gridDim.x) * blockDim.x) >> 5;
-    const uint32_t mask = a.sync_mask;
-
-    float s[M];
-#pragma unroll
-    for (int m = 0; m < M; ++m) s[m] = CLIP ? __ldg(a.clip_scale + m) : 1.0f;
-
-    for (int64_t c = warp; c < n_chunks; c += n_warps) {
-        const int64_t e = c * kSyncChunk + 4 * lane;
-        float g[M][4];
-#pragma unroll
-        for (int m = 0; m < M; ++m) to_array(ld_grad<GDT>(a.grads, m * n + e), g[m]);
-
-        if constexpr (BASE == MTDAO_BASE_ADOPT) {
-            // v first; g becomes the normalised, clamped gradient.
-            {
-                float v[M][4];
-                float *p = a.arena + (1 + N) * a.stride;
-                load_replicas<M>(p, n, e, v);
-#pragma unroll
-                for (int m = 0; m < M; ++m)
-#pragma unroll
-                    for (int k = 0; k < 4; ++k) {
-                        const float gr = g[m][k];
-                        v[m][k] = fmaf(a.sc.c2, fmaf(gr, gr, -v[m][k]), v[m][k]);
-                        float gn = gr / (sqrtf(v[m][k]) + a.sc.eps);
-                        gn = gn > a.sc.clip_c ? a.sc.clip_c : (gn < -a.sc.clip_c ? -a.sc.clip_c : gn);
-                        g[m][k] = gn;
-                    }
-                store_replicas<M>(p, n, e, v, (mask >> (1 + N)) & 1u);
-            }
-            float d[M][4];
-#pragma unroll
-            for (int m = 0; m < M; ++m)
-#pragma unroll
-                for (int k = 0; k < 4; ++k) d[m][k] = a.sc.cg * g[m][k];
-#pragma unroll
-            for (int j = 0; j < N; ++j) {
-                float u[M][4];
-                float *p = a.arena + (1 + j) * a.stride;
-                load_replicas<M>(p, n, e, u);
-#pragma unroll
-                for (int m = 0; m < M; ++m)
-#pragma unroll
-                    for (int k = 0; k < 4; ++k) {
-                        u[m][k] = fmaf(a.sc.c1[j], g[m][k] - u[m][k], u[m][k]);
-                        d[m][k] = fmaf(a.sc.k[j], u[m][k], d[m][k]);
-                    }
-                store_replicas<M>(p, n, e, u, (mask >> (1 + j)) & 1u);
-            }
-            float x[M][4];
-            load_replicas<M>(a.arena, n, e, x);
-#pragma unroll
-            for (int m = 0; m < M; ++m)
-#pragma unroll
-                for (int k = 0; k < 4; ++k) x[m][k] = fmaf(a.sc.neg_lr, d[m][k], x[m][k]);
-            store_replicas<M>(a.arena, n, e, x, mask & 1u);
-        } else {
-            // Adam / SGDM: momenta of the clipped gradient g * s[m], then
-            // (Adam) v of the raw gradient and the denominator, then x.
-            float num[M][4];
-#pragma unroll
-            for (int m = 0; m < M; ++m)
-#pragma unroll
-                for (int k = 0; k < 4; ++k) num[m][k] = a.sc.cg * __fmul_rn(g[m][k], s[m]);
-#pragma unroll
-            for (int j = 0; j < N; ++j) {
-                float u[M][4];
-                float *p = a.arena + (1 + j) * a.stride;
-                load_replicas<M>(p, n, e, u);
-#pragma unroll
-                for (int m = 0; m < M; ++m)
-#pragma unroll
-                    for (int k = 0; k < 4; ++k) {
-                        u[m][k] = fmaf(a.sc.c1[j], __fmul_rn(g[m][k], s[m]) - u[m][k], u[m][k]);
-                        num[m][k] = fmaf(a.sc.k[j], u[m][k], num[m][k]);
-                    }
-                store_replicas<M>(p, n, e, u, (mask >> (1 + j)) & 1u);
-            }
-            if constexpr (BASE == MTDAO_BASE_ADAM) {
-                float v[M][4];
-                float *p = a.arena + (1 + N) * a.stride;
-                load_replicas<M>(p, n, e, v);
-#pragma unroll
-                for (int m = 0; m < M; ++m)
-#pragma unroll
-                    for (int k = 0; k < 4; ++k) {
-                        const float gr = g[m][k];
-                        v[m][k] = fmaf(a.sc.c2, fmaf(gr, gr, -v[m][k]), v[m][k]);
-                        num[m][k] = num[m][k] / fmaf(sqrtf(v[m][k]), a.sc.sv, a.sc.eps);
-                    }
-                store_replicas<M>(p, n, e, v, (mask >> (1 + N)) & 1u);
-            }
-            float x[M][4];
-            load_replicas<M>(a.arena, n, e, x);
-#pragma unroll
-            for (int m = 0; m < M; ++m)
-#pragma unroll
-                for (int k = 0; k < 4; ++k) x[m][k] = fmaf(a.sc.neg_lr, num[m][k], x[m][k]);
-            store_replicas<M>(a.arena, n, e, x, mask & 1u);
-        }
-    }
-}
-
 // ---------------------------------------------------------------- launch helpers
 
 // Persistent grid: as many blocks as fit on the device at once, but never
@@ -330,15 +182,6 @@ cudaError_t launch_step_t(const StepArgs &a, int num_sms, cudaStream_t stream) {
     return cudaGetLastError();
 }
 
-template <int BASE, int N, int GDT, bool CLIP, int M>
-cudaError_t launch_step_sync_t(const StepArgs &a, int num_sms, cudaStream_t stream) {
-    auto kernel = step_sync_kernel<BASE, N, GDT, CLIP, M>;
-    static const int per_sm = blocks_per_sm(kernel);
-    const int grid = persistent_grid(per_sm, num_sms, a.n_padded / kSyncChunk);
-    kernel<<<grid, kThreads, 0, stream>>>(a);
-    return cudaGetLastError();
-}
-
 // Dispatch over N, gradient dtype and clipping for one base.
 template <int BASE>
 cudaError_t launch_step_base(int n_mom, int gdt, bool clip, const StepArgs &a, int num_sms,
@@ -360,38 +203,6 @@ cudaError_t launch_step_base(int n_mom, int gdt, bool clip, const StepArgs &a, i
             return cudaErrorInvalidValue;
     }
 #undef MTDAO_STEP_CASE
-}
-
-template <int BASE, int N, int GDT, bool CLIP>
-cudaError_t launch_step_sync_m(const StepArgs &a, int num_sms, cudaStream_t st) {
-    switch (a.M) {
-        case 2: return launch_step_sync_t<BASE, N, GDT, CLIP, 2>(a, num_sms, st);
-        case 4: return launch_step_sync_t<BASE, N, GDT, CLIP, 4>(a, num_sms, st);
-        case 8: return launch_step_sync_t<BASE, N, GDT, CLIP, 8>(a, num_sms, st);
-        default: return cudaErrorNotSupported;
-    }
-}
-
-template <int BASE>
-cudaError_t launch_step_sync_base(int n_mom, int gdt, bool clip, const StepArgs &a, int num_sms,
-                                  cudaStream_t st) {
-#define MTDAO_SYNC_CASE(NN)                                                                  \
-    case NN:                                                                                 \
-        if (gdt == MTDAO_F32)                                                                \
-            return clip ? launch_step_sync_m<BASE, NN, MTDAO_F32, true>(a, num_sms, st)      \
-                        : launch_step_sync_m<BASE, NN, MTDAO_F32, false>(a, num_sms, st);    \
-        return clip ? launch_step_sync_m<BASE, NN, MTDAO_BF16, true>(a, num_sms, st)         \
-                    : launch_step_sync_m<BASE, NN, MTDAO_BF16, false>(a, num_sms, st);
-    if constexpr (BASE == MTDAO_BASE_ADOPT) clip = false;
-    switch (n_mom) {
-        MTDAO_SYNC_CASE(1)
-        MTDAO_SYNC_CASE(2)
-        MTDAO_SYNC_CASE(3)
-        MTDAO_SYNC_CASE(4)
-        default:
-            return cudaErrorInvalidValue;
-    }
-#undef MTDAO_SYNC_CASE
 }
 
 }  // namespace mtdao
