@@ -333,6 +333,21 @@ def run_ours(args):
     sync_bytes = W.bytes_per_sync(w, n_states)
     sync_gbs = sync_bytes / (statistics.median(sync_ms) / 1e3) / 1e9
 
+    # the same average with the cross-worker diagnostics formed in its pass
+    stats_ms = []
+    if M <= 8:
+        stats_out = torch.empty((n_states, 2 + 2 * M), dtype=torch.float64, device="cuda")
+        for i in range(6):
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            if flush is not None:
+                flush.fill_(1.0)
+            a.record(stream)
+            P.mtdao_sync_stats(eng.h, all_mask, stats_out.data_ptr())
+            b.record(stream)
+            torch.cuda.synchronize()
+            if i >= 2:
+                stats_ms.append(a.elapsed_time(b))
+
     # end to end through the host-buffer C-ABI call
     e2e = None
     if not args.no_e2e and args.e2e_rounds > 0:
@@ -395,6 +410,10 @@ def run_ours(args):
                              "launches_per_round": len(sync_steps) // args.steps},
         "sync_kernel": {"ms_median": statistics.median(sync_ms), "bytes": sync_bytes, "gbs": sync_gbs,
                         "frac": sync_gbs / peak, "states": n_states},
+        "sync_stats_kernel": ({"ms_median": statistics.median(stats_ms),
+                               "gbs": sync_bytes / (statistics.median(stats_ms) / 1e3) / 1e9,
+                               "frac": sync_bytes / (statistics.median(stats_ms) / 1e3) / 1e9 / peak}
+                              if stats_ms else None),
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                      "frac": achieved / peak, "traffic": traffic, "peak_kind": peak_kind,
                      "kernel": "step_kernel (local step, no sync)"},

@@ -220,6 +220,24 @@ int mtdao_step_host(mtdao_handle h, const void *grads_host, int32_t grad_dtype, 
  */
 int mtdao_sync(mtdao_handle h, uint32_t mask);
 
+/*
+ * mtdao_sync plus the paper's cross-worker diagnostics (section 4.1, "Other
+ * Metrics"), formed in the same pass over the replicas at no extra state
+ * traffic.  For every state s in mask, in increasing state order, stats_dev
+ * (device, caller-owned, popcount(mask) * (2 + 2M) doubles) receives, from
+ * the replicas before they are averaged and their fp32 mean s_bar:
+ *   [0]              (1/M) sum_m ||s_m - s_bar||^2   cross-worker variance
+ *   [1]              ||s_bar||^2
+ *   [2 + m]          ||s_m||^2                        m = 0..M-1
+ *   [2 + M + m]      <s_m, s_bar>                     (cosine = [2+M+m] /
+ *                                                      sqrt([2+m] * [1]))
+ * The averaged states are bit-identical to mtdao_sync's.  Sums are
+ * fixed-order (bit-reproducible).  Requires M <= 8; with M = 1 the states
+ * are left as they are and only the diagnostics are written.  A workspace
+ * is allocated on the first call.
+ */
+int mtdao_sync_stats(mtdao_handle h, uint32_t mask, double *stats_dev);
+
 /* Mask of states due at the end of the next step (mtdao_due_mask at t). */
 int mtdao_sync_due(mtdao_handle h, uint32_t *mask_out);
 

@@ -135,6 +135,32 @@ void mto_sync(const mto_cfg *c, int M, long long n, unsigned mask,
         mto_mean_over_workers(M, n, v);
 }
 
+/*
+ * Cross-worker diagnostics of one state s[M][n] (section 4.1, "Other
+ * Metrics"), from the definitions, before any averaging:
+ *   out[0]           (1/M) sum_m ||s_m - s_bar||^2   (cross-worker variance)
+ *   out[1]           ||s_bar||^2
+ *   out[2 + m]       ||s_m||^2
+ *   out[2 + M + m]   <s_m, s_bar>   (with the norms: cosine similarity)
+ * where s_bar = E_m[s] is the worker mean.
+ */
+void mto_state_stats(int M, long long n, const double *s, double *out)
+{
+    for (int k = 0; k < 2 + 2 * M; ++k) out[k] = 0.0;
+    for (long long i = 0; i < n; ++i) {
+        double sum = 0.0;
+        for (int m = 0; m < M; ++m) sum += s[(long long)m * n + i];
+        double mean = sum / (double)M;
+        out[1] += mean * mean;
+        for (int m = 0; m < M; ++m) {
+            double v = s[(long long)m * n + i];
+            out[0] += (v - mean) * (v - mean) / (double)M;
+            out[2 + m] += v * v;
+            out[2 + M + m] += v * mean;
+        }
+    }
+}
+
 /* ||g^m||_2 of one worker's flattened gradient, summed in index order. */
 double mto_grad_norm(long long n, const double *g)
 {

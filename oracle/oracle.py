@@ -95,6 +95,8 @@ def _load():
             lib.mto_adopt_clip_bound.restype = ctypes.c_double
             lib.mto_mean_over_workers.argtypes = [ctypes.c_int, ctypes.c_longlong, dp]
             lib.mto_mean_over_workers.restype = None
+            lib.mto_state_stats.argtypes = [ctypes.c_int, ctypes.c_longlong, dp, dp]
+            lib.mto_state_stats.restype = None
             _lib = lib
     return _lib
 
@@ -197,6 +199,16 @@ def grad_norm(g: np.ndarray) -> float:
 
 def adopt_clip_bound(t: int) -> float:
     return float(_load().mto_adopt_clip_bound(int(t)))
+
+
+def state_stats(s: np.ndarray) -> np.ndarray:
+    """Cross-worker diagnostics of an ``[M][n]`` state (see mto_state_stats):
+    [variance, ||mean||^2, ||s_m||^2 (M), <s_m, mean> (M)]."""
+    s = np.ascontiguousarray(s, np.float64)
+    M = s.shape[0]
+    out = np.zeros(2 + 2 * M, np.float64)
+    _load().mto_state_stats(M, s.size // M, _ptr(s), _ptr(out))
+    return out
 
 
 def mean_over_workers(s: np.ndarray) -> np.ndarray:

@@ -82,6 +82,7 @@ def _load():
                                            ctypes.c_uint32]),
         "mtdao_sync": (ctypes.c_int, [H, ctypes.c_uint32]),
         "mtdao_sync_due": (ctypes.c_int, [H, ctypes.POINTER(ctypes.c_uint32)]),
+        "mtdao_sync_stats": (ctypes.c_int, [H, ctypes.c_uint32, ctypes.c_void_p]),
         "mtdao_grad_sqnorm": (ctypes.c_int, [H, ctypes.c_void_p, ctypes.c_int32, ctypes.c_void_p]),
         "mtdao_grad_sqnorm_static": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_int32, ctypes.c_int32,
                                                     ctypes.c_int64, ctypes.c_void_p, ctypes.c_void_p]),
@@ -218,6 +219,10 @@ def mtdao_sync(h, mask: int) -> None:
     _check(lib.mtdao_sync(h, mask), h)
 
 
+def mtdao_sync_stats(h, mask: int, stats_dev_ptr: int) -> None:
+    _check(lib.mtdao_sync_stats(h, mask, ctypes.c_void_p(stats_dev_ptr)), h)
+
+
 def mtdao_sync_due(h) -> int:
     m = ctypes.c_uint32()
     _check(lib.mtdao_sync_due(h, ctypes.byref(m)), h)
@@ -336,6 +341,15 @@ class MTDAO:
 
     def sync_due(self) -> int:
         return mtdao_sync_due(self.h)
+
+    def sync_stats(self, mask: int):
+        """Average the masked states and return their diagnostics as a
+        device tensor [n_masked][2 + 2M] (see mtdao_sync_stats)."""
+        import torch
+        k = bin(mask).count("1")
+        out = torch.empty((k, 2 + 2 * self.M), dtype=torch.float64, device="cuda")
+        mtdao_sync_stats(self.h, mask, out.data_ptr())
+        return out
 
     def state_ptr(self, state: int, replica: int) -> int:
         return mtdao_get_state_ptr(self.h, state, replica)

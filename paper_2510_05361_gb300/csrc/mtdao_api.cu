@@ -76,6 +76,8 @@ struct mtdao_ctx {
     double *norm_out = nullptr;       // [M]
     double *norm_partial = nullptr;   // [M][norm_blocks]
     int norm_blocks = 1;
+    double *stats_partial = nullptr;  // mtdao_sync_stats workspace (allocated on first use)
+    size_t stats_cap = 0;
     // host-gradient staging (mtdao_step_host)
     void *staging[2] = {nullptr, nullptr};
     size_t staging_bytes = 0;
@@ -234,6 +236,7 @@ void release(mtdao_ctx *h) {
     if (h->clip_scale) cudaFree(h->clip_scale);
     if (h->norm_out) cudaFree(h->norm_out);
     if (h->norm_partial) cudaFree(h->norm_partial);
+    if (h->stats_partial) cudaFree(h->stats_partial);
 }
 
 int check_handle(mtdao_ctx *h) {
@@ -539,6 +542,37 @@ extern "C" int mtdao_sync(mtdao_handle h, uint32_t mask) {
     if (mask == 0 || h->M == 1) return MTDAO_OK;
     if (int rc = select_device(h)) return rc;
     return enqueue_sync(h, mask);
+}
+
+extern "C" int mtdao_sync_stats(mtdao_handle h, uint32_t mask, double *stats_dev) {
+    if (int rc = check_handle(h)) return rc;
+    if (stats_dev == nullptr) return set_error(h, MTDAO_ERR_INVALID, "stats is NULL");
+    if (mask >> h->n_states) return set_error(h, MTDAO_ERR_INVALID, "sync mask 0x%x has bits beyond "
+                                              "the %d states", mask, h->n_states);
+    if (h->M > 8) return set_error(h, MTDAO_ERR_INVALID, "diagnostics support M <= 8 (M = %d)", h->M);
+    if (mask == 0) return MTDAO_OK;
+    if (int rc = select_device(h)) return rc;
+    if (h->stats_partial == nullptr) {
+        const size_t cap = sync_stats_partial_capacity(h->num_sms, h->n_states, h->M);
+        cudaError_t e = cudaMalloc(reinterpret_cast<void **>(&h->stats_partial), cap * sizeof(double));
+        if (e != cudaSuccess) {
+            cudaGetLastError();
+            h->stats_partial = nullptr;
+            return set_error(h, MTDAO_ERR_OOM, "diagnostics workspace: %s", cudaGetErrorString(e));
+        }
+        h->stats_cap = cap;
+    }
+    SyncArgs a;
+    std::memset(&a, 0, sizeof a);
+    a.arena = h->arena;
+    a.n_padded = h->n_padded;
+    a.stride = static_cast<int64_t>(h->M) * h->n_padded;
+    a.M = h->M;
+    for (int s = 0; s < h->n_states; ++s)
+        if (mask & (1u << s)) a.sel[a.n_sel++] = s;
+    cudaError_t e = launch_sync_stats(a, h->num_sms, h->stats_partial, h->stats_cap, stats_dev, h->stream);
+    if (e != cudaSuccess) return cuda_fail(h, e, "sync with diagnostics launch");
+    return MTDAO_OK;
 }
 
 extern "C" int mtdao_sync_due(mtdao_handle h, uint32_t *mask_out) {

@@ -64,6 +64,14 @@ cudaError_t launch_step_sync(int base, int n_mom, int grad_dtype, bool clip, con
 // Replace each selected state by its mean over the M replicas.
 cudaError_t launch_sync(const SyncArgs &a, int num_sms, cudaStream_t stream);
 
+// launch_sync plus the cross-worker diagnostics of every selected state:
+// stats[sel * (2 + 2M) + q], q as documented for mtdao_sync_stats.  Needs a
+// workspace of sync_stats_partial_capacity() doubles; M must be 1..8
+// (cudaErrorNotSupported otherwise).
+size_t sync_stats_partial_capacity(int num_sms, int n_states, int M);
+cudaError_t launch_sync_stats(const SyncArgs &a, int num_sms, double *partial, size_t partial_cap,
+                              double *stats, cudaStream_t stream);
+
 // Per-replica sum of squares of the gradient: partial sums into
 // partial[M][blocks_per_replica], then out[m] (double) and, when
 // clip_scale != nullptr, clip_scale[m] = min(1, rho / (sqrt(out[m]) + 1e-6)).

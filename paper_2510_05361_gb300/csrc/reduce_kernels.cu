@@ -125,7 +125,142 @@ __global__ void __launch_bounds__(kNormThreads) sqnorm_finalize_kernel(const dou
     }
 }
 
+// ---------------------------------------------------------------- sync + diagnostics
+
+// fp32 accumulator with Kahan compensation; value() folds the compensation
+// in at double precision.
+struct Kahan {
+    float s = 0.0f, c = 0.0f;
+    __device__ __forceinline__ void add(float y) {
+        y -= c;
+        const float t = s + y;
+        c = (t - s) - y;
+        s = t;
+    }
+    __device__ __forceinline__ double value() const {
+        return static_cast<double>(s) - static_cast<double>(c);
+    }
+};
+
+// Replica average of the selected states (exactly as sync_kernel) plus, in
+// the same pass over the M replicas, per state and block the partial sums of
+//   q = 0          sum_m (s_m - s_bar)^2        (cross-worker variance * M)
+//   q = 1          s_bar^2
+//   q = 2 + m      s_m^2
+//   q = 2 + M + m  s_m * s_bar
+// written to partial[(sel * gridDim.x + block) * Q + q], Q = 2 + 2M.  s_bar
+// is the fp32 mean that is stored.  With M = 1 nothing is stored (there is
+// nothing to average) but the sums are still formed.
+template <int M>
+__global__ void __launch_bounds__(kThreads) sync_stats_kernel(const SyncArgs a, double *partial) {
+    constexpr int Q = 2 + 2 * M;
+    float *base = a.arena + static_cast<int64_t>(a.sel[blockIdx.y]) * a.stride;
+    const int64_t n = a.n_padded;
+    const int64_t nv = n / 4;
+    Kahan acc[Q];
+    for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < nv;
+         i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+        const int64_t e = 4 * i;
+        float r[M][4];
+#pragma unroll
+        for (int m = 0; m < M; ++m) to_array(ld_state(base + m * n + e), r[m]);
+        float mean[4];
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+            float d = 0.0f;
+#pragma unroll
+            for (int m = 1; m < M; ++m) d += r[m][k] - r[0][k];
+            mean[k] = r[0][k] + d / static_cast<float>(M);
+        }
+        float q[Q];
+#pragma unroll
+        for (int j = 0; j < Q; ++j) q[j] = 0.0f;
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+            q[1] = fmaf(mean[k], mean[k], q[1]);
+#pragma unroll
+            for (int m = 0; m < M; ++m) {
+                const float dv = r[m][k] - mean[k];
+                q[0] = fmaf(dv, dv, q[0]);
+                q[2 + m] = fmaf(r[m][k], r[m][k], q[2 + m]);
+                q[2 + M + m] = fmaf(r[m][k], mean[k], q[2 + M + m]);
+            }
+        }
+#pragma unroll
+        for (int j = 0; j < Q; ++j) acc[j].add(q[j]);
+        if constexpr (M > 1) {
+            const float4 mv = from_array(mean);
+#pragma unroll
+            for (int m = 0; m < M; ++m) st_state(base + m * n + e, mv);
+        }
+    }
+    __shared__ double part[Q][kThreads / 32];
+    const int w = threadIdx.x >> 5, l = threadIdx.x & 31;
+#pragma unroll
+    for (int j = 0; j < Q; ++j) {
+        const double v = warp_sum(acc[j].value());
+        if (l == 0) part[j][w] = v;
+    }
+    __syncthreads();
+    if (threadIdx.x < Q) {
+        double total = 0.0;
+        for (int i = 0; i < static_cast<int>(blockDim.x >> 5); ++i) total += part[threadIdx.x][i];
+        partial[(static_cast<int64_t>(blockIdx.y) * gridDim.x + blockIdx.x) * Q + threadIdx.x] = total;
+    }
+}
+
+// stats[sel * Q + q] = sum over blocks of partial (in block order); q = 0 is
+// divided by M (the variance is a mean over workers).
+__global__ void sync_stats_finalize_kernel(const double *partial, int blocks, int Q, int M,
+                                           double *stats) {
+    const int sel = blockIdx.x, q = threadIdx.x;
+    if (q >= Q) return;
+    double total = 0.0;
+    for (int b = 0; b < blocks; ++b) total += partial[(static_cast<int64_t>(sel) * blocks + b) * Q + q];
+    stats[sel * Q + q] = q == 0 ? total / M : total;
+}
+
+template <int M>
+cudaError_t launch_sync_stats_t(const SyncArgs &a, int num_sms, double *partial, size_t partial_cap,
+                                double *stats, cudaStream_t stream) {
+    constexpr int Q = 2 + 2 * M;
+    static const int per_sm = blocks_per_sm(sync_stats_kernel<M>);
+    const int64_t nv = a.n_padded / 4;
+    int64_t gx = static_cast<int64_t>(per_sm) * num_sms / a.n_sel;
+    const int64_t need = (nv + kThreads - 1) / kThreads;
+    if (gx > need) gx = need;
+    if (gx < 1) gx = 1;
+    if (static_cast<size_t>(gx) * a.n_sel * Q > partial_cap) return cudaErrorInvalidValue;
+    dim3 grid(static_cast<unsigned>(gx), static_cast<unsigned>(a.n_sel));
+    sync_stats_kernel<M><<<grid, kThreads, 0, stream>>>(a, partial);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    sync_stats_finalize_kernel<<<a.n_sel, 32, 0, stream>>>(partial, static_cast<int>(gx), Q, M, stats);
+    return cudaGetLastError();
+}
+
 }  // namespace
+
+size_t sync_stats_partial_capacity(int num_sms, int n_states, int M) {
+    // at most 16 resident blocks per SM of 256 threads, split over the states
+    return static_cast<size_t>(16 * num_sms + n_states) * (2 + 2 * M);
+}
+
+cudaError_t launch_sync_stats(const SyncArgs &a, int num_sms, double *partial, size_t partial_cap,
+                              double *stats, cudaStream_t stream) {
+    if (a.n_sel <= 0) return cudaSuccess;
+    switch (a.M) {
+        case 1: return launch_sync_stats_t<1>(a, num_sms, partial, partial_cap, stats, stream);
+        case 2: return launch_sync_stats_t<2>(a, num_sms, partial, partial_cap, stats, stream);
+        case 3: return launch_sync_stats_t<3>(a, num_sms, partial, partial_cap, stats, stream);
+        case 4: return launch_sync_stats_t<4>(a, num_sms, partial, partial_cap, stats, stream);
+        case 5: return launch_sync_stats_t<5>(a, num_sms, partial, partial_cap, stats, stream);
+        case 6: return launch_sync_stats_t<6>(a, num_sms, partial, partial_cap, stats, stream);
+        case 7: return launch_sync_stats_t<7>(a, num_sms, partial, partial_cap, stats, stream);
+        case 8: return launch_sync_stats_t<8>(a, num_sms, partial, partial_cap, stats, stream);
+        default: return cudaErrorNotSupported;
+    }
+}
 
 cudaError_t launch_sync(const SyncArgs &a, int num_sms, cudaStream_t stream) {
     if (a.n_sel <= 0 || a.M <= 1) return cudaSuccess;

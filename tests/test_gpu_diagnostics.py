@@ -1,0 +1,107 @@
+"""Sync with diagnostics (mtdao_sync_stats) against the oracle's definitions
+of the paper's cross-worker metrics (section 4.1), and bit-equality of the
+averaged states with the plain sync."""
+import numpy as np
+import pytest
+
+torch = pytest.importorskip("torch")
+
+from oracle.oracle import state_stats
+from parity_util import workload_dict
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def P():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    import paper_2510_05361_gb300 as P
+    P.load()
+    return P
+
+
+def _fill(eng, rng, spread):
+    vals = {}
+    for s in range(eng.n_states):
+        common = rng.standard_normal(eng.n_padded).astype(np.float32)
+        arr = (common[None, :] + spread * rng.standard_normal((eng.M, eng.n_padded))).astype(np.float32)
+        if s == eng.n_states - 1:
+            arr = np.abs(arr)
+        eng.state_view(s).copy_(torch.from_numpy(arr).cuda())
+        vals[s] = arr
+    return vals
+
+
+@pytest.mark.parametrize("M", [1, 2, 3, 4, 8])
+def test_sync_stats_match_oracle_and_plain_sync(P, M):
+    shapes = [70001, 999, 4096]
+    w = workload_dict(shapes, M, betas=(0.9, 0.99))
+    a = P.MTDAO(w["opt"], M, shapes)
+    b = P.MTDAO(w["opt"], M, shapes)
+    rng = np.random.default_rng(M)
+    vals = _fill(a, rng, spread=0.05)
+    for s, arr in vals.items():
+        b.state_view(s).copy_(torch.from_numpy(arr).cuda())
+    mask = 0b1101                                 # x, u2, v
+    stats = a.sync_stats(mask).cpu().numpy()
+    b.sync(mask)
+    again = P.MTDAO(w["opt"], M, shapes)
+    for s, arr in vals.items():
+        again.state_view(s).copy_(torch.from_numpy(arr).cuda())
+    stats2 = again.sync_stats(mask).cpu().numpy()
+    torch.cuda.synchronize()
+    assert np.array_equal(stats, stats2)          # fixed-order sums
+    sel = [s for s in range(a.n_states) if (mask >> s) & 1]
+    assert stats.shape == (len(sel), 2 + 2 * M)
+    for row, s in zip(stats, sel):
+        ref = state_stats(vals[s].astype(np.float64))
+        err = np.abs(row - ref) / np.maximum(np.abs(ref), 1e-30)
+        assert np.all(err[1:] <= 1e-5), (s, err)
+        if M > 1:
+            assert err[0] <= 1e-5, (s, err[0])
+        else:
+            assert row[0] == 0.0
+    for s in range(a.n_states):
+        ga = a.state_view(s).cpu().numpy()
+        gb = b.state_view(s).cpu().numpy()
+        assert np.array_equal(ga.view(np.uint32), gb.view(np.uint32)), s
+    for e in (a, b, again):
+        e.close()
+
+
+def test_sync_stats_cosine_and_variance_during_training(P):
+    """After a few local steps from a common start, the cosine between each
+    worker's momentum and the mean momentum is in (0, 1] and the variance
+    vanishes after the momenta are averaged."""
+    M = 4
+    w = workload_dict([50000], M, betas=(0.9,), px=0, pu=0, pv=0)
+    eng = P.MTDAO(w["opt"], M, w["shapes"])
+    eng.set_params(torch.zeros(eng.n_padded, device="cuda"))
+    gen = torch.Generator(device="cuda").manual_seed(3)
+    common = torch.randn(eng.n_padded, device="cuda", generator=gen)
+    for t in range(8):
+        g = common[None, :] + 0.5 * torch.randn((M, eng.n_padded), device="cuda", generator=gen)
+        eng.step(g.contiguous(), 1e-3, 0)
+    st = eng.sync_stats(0b10).cpu().numpy()[0]     # u1
+    cos = st[2 + M:] / np.sqrt(st[2:2 + M] * st[1])
+    assert np.all(cos > 0.5) and np.all(cos <= 1.0 + 1e-6)
+    assert st[0] > 0
+    st2 = eng.sync_stats(0b10).cpu().numpy()[0]
+    assert st2[0] <= 1e-10 * st2[1]
+    eng.close()
+
+
+def test_sync_stats_rejects_large_M_and_bad_masks(P):
+    w = workload_dict([1024], 9, betas=(0.9,))
+    eng = P.MTDAO(w["opt"], 9, w["shapes"])
+    out = torch.zeros(64, dtype=torch.float64, device="cuda")
+    with pytest.raises(P.MTDAOError) as e:
+        P.mtdao_sync_stats(eng.h, 1, out.data_ptr())
+    assert e.value.code == P.ERR_INVALID
+    eng.close()
+    w = workload_dict([1024], 2, betas=(0.9,))
+    eng = P.MTDAO(w["opt"], 2, w["shapes"])
+    with pytest.raises(P.MTDAOError):
+        P.mtdao_sync_stats(eng.h, 1 << 7, out.data_ptr())
+    eng.close()

@@ -30,8 +30,9 @@ MUTATIONS = {
     "adopt_normalises_with_old_v": ("double g_hat = g / (sqrt(v_new) + c->eps);",
                                     "double g_hat = g / (sqrt(c->beta2 * v_new) + c->eps);"),
     "adopt_clamp_missing": ("if (g_tilde > ct) g_tilde = ct;", "if (0) g_tilde = ct;"),
-    "mean_divides_by_M_minus_1": ("double mean = sum / (double)M;",
-                                  "double mean = sum / (double)(M > 1 ? M - 1 : 1);"),
+    "mean_divides_by_M_minus_1": (
+        "double mean = sum / (double)M;\n        for (int m = 0; m < M; ++m)\n            s[",
+        "double mean = sum / (double)(M > 1 ? M - 1 : 1);\n        for (int m = 0; m < M; ++m)\n            s["),
     "sync_phase_off_by_one": (
         "    if (divides(c->period_x, t)) mask |= bit_x();\n    for (int j = 0; j < c->n_mom; ++j)\n"
         "        if (divides(c->period_u[j], t)) mask |= bit_u(j);",
@@ -47,6 +48,9 @@ MUTATIONS = {
         "        delta += c->omega[j] * u_new;\n    }\n    x[k] = x[k] - lr * delta;\n    return x[k];\n}\n\n/*\n * One"),
     "v_sync_skipped": ("    if (c->base != MTO_SGDM && (mask & bit_v(c)))\n        mto_mean_over_workers(M, n, v);",
                        "    if (0)\n        mto_mean_over_workers(M, n, v);"),
+    "variance_over_M_minus_1": ("out[0] += (v - mean) * (v - mean) / (double)M;",
+                                "out[0] += (v - mean) * (v - mean) / (double)(M - 1);"),
+    "dot_with_worker_instead_of_mean": ("out[2 + M + m] += v * mean;", "out[2 + M + m] += v * v;"),
 }
 
 

@@ -435,3 +435,28 @@ def test_invalid_pairings_rejected():
         Oracle(cfg("adopt", (0.9,), clip="global_norm"), 1, 4).step(0, 1e-3, np.zeros((1, 4)))
     with pytest.raises(ValueError):
         Oracle(cfg("adam", (0.9,), clip="elementwise"), 1, 4).step(0, 1e-3, np.zeros((1, 4)))
+
+
+# ----------------------------------------------------- diagnostics pins
+
+def test_state_stats_against_numpy_and_closed_forms():
+    """Section 4.1 metrics: cross-worker variance (1/M) sum ||s_m - s_bar||^2,
+    norms and the dot products of each worker with the mean."""
+    from oracle.oracle import state_stats
+    rng = np.random.default_rng(16)
+    M, n = 5, 333
+    s = rng.standard_normal((M, n))
+    out = state_stats(s)
+    mean = s.mean(axis=0)
+    assert abs(out[0] - s.var(axis=0).sum()) < 1e-12 * out[0]
+    assert abs(out[1] - np.dot(mean, mean)) < 1e-12 * out[1]
+    np.testing.assert_allclose(out[2:2 + M], np.linalg.norm(s, axis=1) ** 2, rtol=1e-13)
+    np.testing.assert_allclose(out[2 + M:], s @ mean, rtol=1e-12)
+    # M = 2: variance = ||a - b||^2 / 4
+    two = state_stats(s[:2])
+    assert abs(two[0] - np.sum((s[0] - s[1]) ** 2) / 4) < 1e-12 * two[0]
+    # identical workers: no variance (up to the rounding of the fp64 mean),
+    # every norm and dot equals ||s||^2
+    same = state_stats(np.tile(s[0], (3, 1)))
+    assert 0.0 <= same[0] <= 1e-28 * same[1]
+    np.testing.assert_allclose(same[1:], np.dot(s[0], s[0]), rtol=1e-14)
