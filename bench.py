@@ -52,6 +52,10 @@ def parse_args():
     ap.add_argument("--e2e-rounds", type=int, default=2)
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--sweep", action="store_true",
+                    help="flat-vector sweep: one JSON line per (n, M, N) with step, fused "
+                         "step+sync and sync bandwidth, and the round rate for H in {1, 8, 64}")
+    ap.add_argument("--sweep-log2n", default="20,24,27,30")
     return ap.parse_args()
 
 
@@ -430,10 +434,84 @@ def run_ours(args):
     return 0
 
 
+def run_sweep(args):
+    """Flat fp32 vector n = 2^k, M in {1,2,4,8}, N in {1..4} (Adam, f32
+    gradients).  Each (n, M, N) point times 6 launches (2 warm-up) of the
+    plain step, the fused step + average of every state, and the standalone
+    average; per H in {1, 8, 64} a round is (H-1) plain steps and one fused
+    step, so its rate follows from those times."""
+    import torch
+
+    import paper_2510_05361_gb300 as P
+    from synth.device import DeviceInputs
+
+    torch.cuda.set_device(int(os.environ.get("LOCAL_RANK", "0")))
+    P.load()
+    peak, peak_kind = hbm_peak()
+    stream = torch.cuda.current_stream()
+
+    def timed(fn, reps=6, skip=2):
+        out = []
+        for i in range(reps):
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record(stream)
+            fn()
+            b.record(stream)
+            torch.cuda.synchronize()
+            if i >= skip:
+                out.append(a.elapsed_time(b))
+        return statistics.median(out)
+
+    for k in [int(v) for v in args.sweep_log2n.split(",")]:
+        for M in (1, 2, 4, 8):
+            for N in (1, 2, 3, 4):
+                w = W.sweep_point(k, M, N, 8)
+                n_states = N + 2
+                need = M * (1 << k) * (4 * n_states + 4) + (4 << 30)
+                free = torch.cuda.mem_get_info()[0]
+                rec = {"sweep": True, "log2_n": k, "M": M, "N": N, "base": "adam", "grad_dtype": "f32"}
+                if need > free:
+                    rec["skipped"] = "needs %.0f GB, %.0f GB free" % (need / 1e9, free / 1e9)
+                    print(json.dumps(rec), flush=True)
+                    continue
+                lay = W.layout(w["shapes"])
+                eng = P.MTDAO(w["opt"], M, w["shapes"], stream=stream.cuda_stream)
+                inputs = DeviceInputs(w, lay, W.GRAD_SEED, W.INIT_SEED)
+                eng.set_params(inputs.init_params())
+                g = inputs.grads(0)
+                all_mask = (1 << n_states) - 1
+                lr = w["opt"]["lr"]
+                t_step = timed(lambda: P.mtdao_step(eng.h, g.data_ptr(), P.F32, lr, 0))
+                t_fused = timed(lambda: P.mtdao_step(eng.h, g.data_ptr(), P.F32, lr, all_mask))
+                t_sync = timed(lambda: P.mtdao_sync(eng.h, all_mask)) if M > 1 else None
+                step_bytes = W.bytes_per_step(w)
+                sync_bytes = W.bytes_per_sync(w, n_states)
+                rec.update({
+                    "step_ms": t_step, "step_gbs": step_bytes / t_step / 1e6,
+                    "step_frac": step_bytes / t_step / 1e6 / peak,
+                    "fused_ms": t_fused, "fused_gbs": step_bytes / t_fused / 1e6,
+                    "fused_frac": step_bytes / t_fused / 1e6 / peak,
+                    "sync_ms": t_sync,
+                    "sync_gbs": (sync_bytes / t_sync / 1e6) if t_sync else None,
+                    "sync_frac": (sync_bytes / t_sync / 1e6 / peak) if t_sync else None,
+                    "peak_gbs": peak, "peak_kind": peak_kind,
+                    "round_params_per_s": {
+                        str(H): M * lay["n_padded"] * H / (((H - 1) * t_step + t_fused) / 1e3)
+                        for H in (1, 8, 64)},
+                })
+                print(json.dumps(rec), flush=True)
+                del g
+                eng.close()
+                torch.cuda.empty_cache()
+    return 0
+
+
 def main():
     args = parse_args()
     if args.impl == "reference":
         return run_reference(args)
+    if args.sweep:
+        return run_sweep(args)
     return run_ours(args)
 
 

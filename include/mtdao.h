@@ -44,7 +44,7 @@
 extern "C" {
 #endif
 
-#define MTDAO_VERSION 1
+#define MTDAO_VERSION 2
 #define MTDAO_MAX_MOM 4          /* largest N supported */
 #define MTDAO_MAX_REPLICAS 64    /* largest M supported */
 
@@ -68,7 +68,8 @@ typedef enum {
     /* Adam/SGDM clip(g, rho): each replica's whole flattened gradient is
      * scaled by min(1, rho / (||g||_2 + 1e-6)); v keeps the raw gradient. */
     MTDAO_CLIP_GLOBAL_NORM = 1,
-    /* ADOPT clip(g-hat, c_t): elementwise clamp to +-c_t, c_t = (t+1)^(1/4). */
+    /* ADOPT clip(g-hat, c_t): elementwise clamp to +-c_t, c_t = (t+1)^(1/4)
+     * (t the 0-based step; see adopt_prev_v for the other ordering). */
     MTDAO_CLIP_ELEMENTWISE = 2
 } mtdao_clip;
 
@@ -103,6 +104,12 @@ typedef struct {
     int64_t period_x;                   /* K_x; 0 = never averaged */
     int64_t period_u[MTDAO_MAX_MOM];    /* K_j; 0 = never */
     int64_t period_v;                   /* K_v; 0 = never (ignored for SGDM) */
+    int32_t adopt_prev_v;               /* ADOPT only.  0 = Algorithm 2 order: normalise
+                                           with the freshly updated v.  1 = the original
+                                           ADOPT order: step 0 only sets v = g_0^2, later
+                                           steps normalise with the previous v, then update
+                                           it.  The clamp bound is c = k^(1/4) for the k-th
+                                           parameter update (1-based) in both orders. */
 } mtdao_config;
 
 typedef struct mtdao_ctx *mtdao_handle;

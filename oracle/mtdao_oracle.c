@@ -37,6 +37,11 @@
  *   - clip(g-hat, c_t) for ADOPT is an elementwise clamp to [-c_t, c_t] with
  *     c_t = (t+1)^(1/4), or no clamp at all.
  *   - ADOPT normalises with the freshly updated v_t (Algorithm 2 order).
+ *     adopt_prev_v=1 selects the ordering of the original ADOPT method
+ *     instead: step 0 only sets v = g_0^2 (no momentum or parameter update),
+ *     and every later step normalises with the previous v before updating
+ *     it; the clamp bound is then c = t^(1/4), t being the 1-based index of
+ *     the parameter update in both orders.
  */
 #include <math.h>
 #include <stddef.h>
@@ -62,6 +67,7 @@ typedef struct {
     long long period_u[MTO_MAX_MOM];/* K_j                                    */
     long long period_v;             /* K_v                                    */
     int sync_phase;                 /* MTO_PHASE_*                            */
+    int adopt_prev_v;               /* ADOPT: original ordering (see above)   */
 } mto_cfg;
 
 /* Number of state vectors per worker: x, u^1..u^N and (Adam/ADOPT) v. */
@@ -219,12 +225,24 @@ static double adopt_element(const mto_cfg *c, long long t, double lr, double g,
     double sum_omega = 0.0;
     for (int j = 0; j < c->n_mom; ++j) sum_omega += c->omega[j];
 
-    double v_new = c->beta2 * v[k] + (1.0 - c->beta2) * g * g;
-    v[k] = v_new;
-    double g_hat = g / (sqrt(v_new) + c->eps);
+    double g_hat;
+    long long update_index = t;           /* 0-based index of this x update */
+    if (c->adopt_prev_v) {
+        if (t == 0) {                     /* v_0 = g_0^2; nothing else moves */
+            v[k] = g * g;
+            return x[k];
+        }
+        g_hat = g / (sqrt(v[k]) + c->eps);
+        v[k] = c->beta2 * v[k] + (1.0 - c->beta2) * g * g;
+        update_index = t - 1;
+    } else {
+        double v_new = c->beta2 * v[k] + (1.0 - c->beta2) * g * g;
+        v[k] = v_new;
+        g_hat = g / (sqrt(v_new) + c->eps);
+    }
     double g_tilde = g_hat;
     if (c->clip_mode == MTO_CLIP_ELEMENTWISE) {
-        double ct = mto_adopt_clip_bound(t);
+        double ct = mto_adopt_clip_bound(update_index);
         if (g_tilde > ct) g_tilde = ct;
         if (g_tilde < -ct) g_tilde = -ct;
     }
@@ -275,6 +293,7 @@ int mto_step(const mto_cfg *c, int M, long long n, long long t, double lr,
      * of the paper. */
     if (c->base == MTO_ADOPT && c->clip_mode == MTO_CLIP_GLOBAL_NORM) return -1;
     if (c->base != MTO_ADOPT && c->clip_mode == MTO_CLIP_ELEMENTWISE) return -1;
+    if (c->base != MTO_ADOPT && c->adopt_prev_v) return -1;
 
     if (c->sync_phase == MTO_PHASE_ALG1)
         mto_sync(c, M, n, mto_due_before_step(c, t), x, u, v);

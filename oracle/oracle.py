@@ -47,6 +47,7 @@ class _Cfg(ctypes.Structure):
         ("period_u", ctypes.c_longlong * _MAX_MOM),
         ("period_v", ctypes.c_longlong),
         ("sync_phase", ctypes.c_int),
+        ("adopt_prev_v", ctypes.c_int),
     ]
 
 
@@ -119,6 +120,7 @@ def make_cfg(cfg: dict) -> _Cfg:
     c.period_x = int(cfg["period_x"])
     c.period_v = int(cfg.get("period_v", 0))
     c.sync_phase = PHASES[cfg.get("sync_phase", "alg1")]
+    c.adopt_prev_v = 1 if cfg.get("adopt_prev_v", False) else 0
     return c
 
 

@@ -47,6 +47,7 @@ class mtdao_config(ctypes.Structure):
         ("period_x", ctypes.c_int64),
         ("period_u", ctypes.c_int64 * MAX_MOM),
         ("period_v", ctypes.c_int64),
+        ("adopt_prev_v", ctypes.c_int32),
     ]
 
 
@@ -149,6 +150,7 @@ def make_config(opt: dict) -> mtdao_config:
     c.sync_phase = PHASES[opt.get("sync_phase", "alg1")]
     c.period_x = int(opt["period_x"])
     c.period_v = int(opt.get("period_v", 0))
+    c.adopt_prev_v = 1 if opt.get("adopt_prev_v", False) else 0
     return c
 
 

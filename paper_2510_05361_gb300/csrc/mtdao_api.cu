@@ -160,6 +160,10 @@ int validate(const mtdao_config *c, int32_t M) {
             break;
         default: return set_error(nullptr, MTDAO_ERR_INVALID, "unknown clip mode %d", c->clip_mode);
     }
+    if (c->adopt_prev_v != 0 && c->adopt_prev_v != 1)
+        return set_error(nullptr, MTDAO_ERR_INVALID, "adopt_prev_v must be 0 or 1");
+    if (c->adopt_prev_v && c->base != MTDAO_BASE_ADOPT)
+        return set_error(nullptr, MTDAO_ERR_INVALID, "adopt_prev_v applies to the ADOPT base only");
     if (c->sync_phase != MTDAO_PHASE_ALG1 && c->sync_phase != MTDAO_PHASE_ALG2_LITERAL)
         return set_error(nullptr, MTDAO_ERR_INVALID, "unknown sync phase %d", c->sync_phase);
     if (c->period_x < 0) return set_error(nullptr, MTDAO_ERR_INVALID, "period_x negative");
@@ -201,9 +205,19 @@ StepScalars step_scalars(const mtdao_config *c, int64_t t, double lr) {
     s.sv = adam_bc ? static_cast<float>(1.0 / std::sqrt(1.0 - std::pow(c->beta2, static_cast<double>(t + 1))))
                    : 1.0f;
     s.eps = static_cast<float>(c->eps);
-    s.clip_c = (c->base == MTDAO_BASE_ADOPT && c->clip_mode == MTDAO_CLIP_ELEMENTWISE)
-                   ? static_cast<float>(std::pow(static_cast<double>(t + 1), 0.25))
+    // k: 1-based index of the parameter update this step makes
+    const bool prev_v = c->base == MTDAO_BASE_ADOPT && c->adopt_prev_v;
+    const int64_t k = prev_v ? t : t + 1;
+    s.clip_c = (c->base == MTDAO_BASE_ADOPT && c->clip_mode == MTDAO_CLIP_ELEMENTWISE && k >= 1)
+                   ? static_cast<float>(std::pow(static_cast<double>(k), 0.25))
                    : INFINITY;
+    s.prev_v = prev_v ? 1 : 0;
+    if (prev_v && t == 0) {
+        // original ADOPT order, step 0: v = g_0^2 and nothing else moves
+        s.c2 = 1.0f;
+        for (int j = 0; j < c->n_mom; ++j) s.c1[j] = 0.0f;
+        s.neg_lr = 0.0f;
+    }
     return s;
 }
 
@@ -286,6 +300,7 @@ extern "C" int mtdao_config_default(mtdao_config *cfg, int32_t base, int32_t n_m
     cfg->sync_phase = MTDAO_PHASE_ALG1;
     cfg->period_x = 32;
     cfg->period_v = base == MTDAO_BASE_SGDM ? 0 : 32;
+    cfg->adopt_prev_v = 0;
     return MTDAO_OK;
 }
 

@@ -29,6 +29,7 @@ struct StepScalars {
     float sv;                        // Adam: 1 / sqrt(1 - beta_2^(t+1)), or 1
     float eps;                       // epsilon
     float clip_c;                    // ADOPT clamp bound c_t (+inf when not clipping)
+    int prev_v;                      // ADOPT: normalise with the previous v (original order)
 };
 
 struct StepArgs {

@@ -63,9 +63,16 @@ __device__ __forceinline__ void update_element(const StepScalars &sc, float g, f
                                                float &x, float *u, float &v) {
     if constexpr (BASE == MTDAO_BASE_ADOPT) {
         // Algorithm 2: second moment from the raw gradient first, then the
-        // normalised and clamped gradient drives every first momentum.
-        v = fmaf(sc.c2, fmaf(g, g, -v), v);
-        float gn = g / (sqrtf(v) + sc.eps);
+        // normalised and clamped gradient drives every first momentum.  In
+        // the original ADOPT order (uniform flag) v is updated after use.
+        float gn;
+        if (sc.prev_v) {
+            gn = g / (sqrtf(v) + sc.eps);
+            v = fmaf(sc.c2, fmaf(g, g, -v), v);
+        } else {
+            v = fmaf(sc.c2, fmaf(g, g, -v), v);
+            gn = g / (sqrtf(v) + sc.eps);
+        }
         gn = gn > sc.clip_c ? sc.clip_c : (gn < -sc.clip_c ? -sc.clip_c : gn);  // keeps NaN
         float delta = sc.cg * gn;
 #pragma unroll

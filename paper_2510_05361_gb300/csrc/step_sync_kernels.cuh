@@ -117,8 +117,14 @@ __global__ void __launch_bounds__(kThreads, 2) step_sync_kernel(const StepArgs a
 #pragma unroll
                     for (int k = 0; k < V; ++k) {
                         const float gr = g[m][k];
-                        v[m][k] = fmaf(a.sc.c2, fmaf(gr, gr, -v[m][k]), v[m][k]);
-                        float gn = gr / (sqrtf(v[m][k]) + a.sc.eps);
+                        float gn;
+                        if (a.sc.prev_v) {
+                            gn = gr / (sqrtf(v[m][k]) + a.sc.eps);
+                            v[m][k] = fmaf(a.sc.c2, fmaf(gr, gr, -v[m][k]), v[m][k]);
+                        } else {
+                            v[m][k] = fmaf(a.sc.c2, fmaf(gr, gr, -v[m][k]), v[m][k]);
+                            gn = gr / (sqrtf(v[m][k]) + a.sc.eps);
+                        }
                         gn = gn > a.sc.clip_c ? a.sc.clip_c : (gn < -a.sc.clip_c ? -a.sc.clip_c : gn);
                         g[m][k] = gn;
                     }

@@ -40,7 +40,7 @@ def test_library_exports_every_declared_symbol(P):
     lib = ctypes.CDLL(P.LIB_PATH)
     missing = [n for n in declared_functions() if not hasattr(lib, n)]
     assert not missing, missing
-    assert P.mtdao_version() == 1
+    assert P.mtdao_version() == 2
 
 
 def test_layout_matches_the_published_convention(P):
@@ -94,6 +94,7 @@ def test_paper_period_counts(P):
     {"base": "adopt", "bias_correction": True}, {"base": "adopt", "clip_mode": "global_norm",
                                                  "bias_correction": False},
     {"clip_mode": "global_norm", "clip_rho": 0.0}, {"beta1": [float("nan"), 0.9]},
+    {"adopt_prev_v": True},
 ])
 def test_invalid_configurations_are_rejected(P, bad):
     opt = _opt()

@@ -149,6 +149,20 @@ def test_adopt_clip_parity(P, clip):
     eng.close()
 
 
+@pytest.mark.parametrize("M", [3, 4, 8])
+@pytest.mark.parametrize("clip", ["elementwise", "none"])
+def test_adopt_original_ordering_parity(P, clip, M):
+    """adopt_prev_v (original ADOPT order): step 0 only initialises v."""
+    w = workload_dict(RAGGED, M, base="adopt", betas=(0.95, 0.999), beta2=0.9999, clip=clip,
+                      px=5, pu=3, pv=4, lr=2.0 ** -8)
+    w["opt"]["adopt_prev_v"] = True
+    eng = gpu_run(P, w, 17)
+    lay = W.layout(w["shapes"])
+    ref = oracle_run(w["opt"], M, np.arange(lay["n_padded"]), 17, lay, w, SEED_G, SEED_I)
+    compare(gpu_states(eng, w["opt"]), ref)
+    eng.close()
+
+
 def test_alg2_literal_phase_parity(P):
     w = workload_dict(RAGGED, 4, base="adopt", betas=(0.95,), beta2=0.9999, px=4, pu=3, pv=5,
                       phase="alg2_literal", lr=2.0 ** -8)

@@ -27,8 +27,12 @@ MUTATIONS = {
     "gradient_term_dropped": ("double combo = (1.0 - sum_omega) * g_hat;", "double combo = 0.0;"),
     "adam_update_sign": ("x[k] = x[k] - lr * delta;\n    return x[k];\n}\n\n/* Algorithm 2",
                          "x[k] = x[k] + lr * delta;\n    return x[k];\n}\n\n/* Algorithm 2"),
-    "adopt_normalises_with_old_v": ("double g_hat = g / (sqrt(v_new) + c->eps);",
-                                    "double g_hat = g / (sqrt(c->beta2 * v_new) + c->eps);"),
+    "adopt_normalises_with_old_v": ("g_hat = g / (sqrt(v_new) + c->eps);",
+                                    "g_hat = g / (sqrt(c->beta2 * v_new) + c->eps);"),
+    "adopt_original_order_uses_new_v": (
+        "        g_hat = g / (sqrt(v[k]) + c->eps);\n        v[k] = c->beta2 * v[k] + (1.0 - c->beta2) * g * g;",
+        "        v[k] = c->beta2 * v[k] + (1.0 - c->beta2) * g * g;\n        g_hat = g / (sqrt(v[k]) + c->eps);"),
+    "adopt_original_order_clamp_index": ("update_index = t - 1;", "update_index = t;"),
     "adopt_clamp_missing": ("if (g_tilde > ct) g_tilde = ct;", "if (0) g_tilde = ct;"),
     "mean_divides_by_M_minus_1": (
         "double mean = sum / (double)M;\n        for (int m = 0; m < M; ++m)\n            s[",

@@ -331,6 +331,41 @@ def test_adopt_constant_gradient_closed_form(clip):
         assert abs(adopt_clip_bound(15) - 2.0) < 1e-15
 
 
+@pytest.mark.parametrize("clip", ["elementwise", "none"])
+def test_adopt_original_ordering_closed_form(clip):
+    """adopt_prev_v: step 0 sets v = g_0^2 and moves nothing else; step t >= 1
+    normalises with the previous v, v_{t-1} = b2^(t-1) g_0^2 + (1 - b2^(t-1)) g^2
+    for a gradient g_0 then constant g, and clamps to +-t^(1/4) at the t-th
+    update.  A small g_0 makes the clamp bind."""
+    betas, om = (0.9, 0.99), (0.4, 0.5)
+    b2, eps = 0.9999, 1e-8
+    c = cfg("adopt", betas, omega=om, beta2=b2, eps=eps, bias=False, clip=clip)
+    c["adopt_prev_v"] = True
+    rng = np.random.default_rng(17)
+    M, n, T = 2, 16, 20
+    g = rng.standard_normal((M, n)) * np.logspace(-4, 1, n)
+    g0 = 1e-3 * g
+    x0 = rng.standard_normal(n)
+    o = Oracle(c, M, n, x0=x0)
+    o.step(0, 0.1, g0)
+    assert np.array_equal(o.v, g0 * g0) and np.all(o.u == 0) and np.all(o.x == x0[None, :])
+    x = np.broadcast_to(x0, (M, n)).copy()
+    hist = []
+    for t in range(1, T):
+        o.step(t, 0.01, g)
+        v_prev = b2 ** (t - 1) * g0 * g0 + (1 - b2 ** (t - 1)) * g * g
+        gh = g / (np.sqrt(v_prev) + eps)
+        if clip == "elementwise":
+            gh = np.clip(gh, -t ** 0.25, t ** 0.25)
+        hist.append(gh)
+        us = [sum((1 - b) * b ** (len(hist) - 1 - k) * hist[k] for k in range(len(hist))) for b in betas]
+        x = x - 0.01 * ((1 - sum(om)) * gh + sum(w * u for w, u in zip(om, us)))
+        assert rel(o.v, b2 ** t * g0 * g0 + (1 - b2 ** t) * g * g) < 1e-12
+    assert rel(o.x, x) < 1e-11
+    if clip == "elementwise":
+        assert np.max(np.abs(hist[0])) == 1.0          # the clamp bound at the first update
+
+
 # ------------------------------------------------------------- sync pins
 
 def test_sync_identity_on_identical_workers():
