@@ -141,7 +141,9 @@ int32_t mtdao_num_states(const mtdao_config *cfg);
 /*
  * Flattened layout of a tensor list: offsets_out[k] (n_tensors entries,
  * caller-owned) and *n_padded_out as described under "Layout" above.
- * MTDAO_ERR_INVALID for a non-positive numel or n_tensors.  No device access.
+ * Zero-size tensors take no space (their offset is that of the next one).
+ * MTDAO_ERR_INVALID for a negative numel, n_tensors < 1 or a list with no
+ * element at all.  No device access.
  */
 int mtdao_plan_layout(const int64_t *tensor_numel, int32_t n_tensors,
                       int64_t *offsets_out, int64_t *n_padded_out);

@@ -53,15 +53,22 @@ class _Cfg(ctypes.Structure):
 
 def build(force: bool = False) -> str:
     """Compile the oracle with gcc (no FMA contraction, no fast-math)."""
+    import fcntl
     os.makedirs(os.path.dirname(_LIB), exist_ok=True)
-    if (not force and os.path.exists(_LIB)
-            and os.path.getmtime(_LIB) >= os.path.getmtime(_SRC)):
+
+    def fresh():
+        return os.path.exists(_LIB) and os.path.getmtime(_LIB) >= os.path.getmtime(_SRC)
+
+    if not force and fresh():
         return _LIB
-    tmp = _LIB + ".%d.tmp" % os.getpid()
-    cmd = ["gcc", "-O2", "-std=c99", "-fPIC", "-shared", "-ffp-contract=off",
-           "-fno-fast-math", _SRC, "-o", tmp, "-lm"]
-    subprocess.run(cmd, check=True)
-    os.replace(tmp, _LIB)
+    with open(os.path.join(os.path.dirname(_LIB), ".lock"), "w") as lock:
+        fcntl.flock(lock, fcntl.LOCK_EX)           # one builder at a time
+        if force or not fresh():
+            tmp = _LIB + ".%d.tmp" % os.getpid()
+            cmd = ["gcc", "-O2", "-std=c99", "-fPIC", "-shared", "-ffp-contract=off",
+                   "-fno-fast-math", _SRC, "-o", tmp, "-lm"]
+            subprocess.run(cmd, check=True)
+            os.replace(tmp, _LIB)
     return _LIB
 
 

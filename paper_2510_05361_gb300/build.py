@@ -8,6 +8,8 @@ and square root, no flush-to-zero, no fast-math.  Run
 from __future__ import annotations
 
 import concurrent.futures as cf
+import contextlib
+import fcntl
 import os
 import shutil
 import subprocess
@@ -47,11 +49,29 @@ def up_to_date() -> bool:
     return all(os.path.getmtime(f) <= t for f in _deps())
 
 
+@contextlib.contextmanager
+def _build_lock():
+    """Serialise concurrent builds (parallel test workers, several ranks)."""
+    os.makedirs(OUT_DIR, exist_ok=True)
+    with open(os.path.join(OUT_DIR, ".lock"), "w") as f:
+        fcntl.flock(f, fcntl.LOCK_EX)
+        try:
+            yield
+        finally:
+            fcntl.flock(f, fcntl.LOCK_UN)
+
+
 def build(force: bool = False, verbose: bool = False, ptxas_info: bool = False) -> str:
     if not force and up_to_date():
         return LIB
+    with _build_lock():
+        if not force and up_to_date():
+            return LIB
+        return _build(verbose, ptxas_info)
+
+
+def _build(verbose: bool, ptxas_info: bool) -> str:
     nvcc = _nvcc()
-    os.makedirs(OUT_DIR, exist_ok=True)
     extra = ["-Xptxas", "-v"] if ptxas_info else []
 
     def compile_one(src):

@@ -317,11 +317,12 @@ extern "C" int mtdao_plan_layout(const int64_t *numel, int32_t n_tensors, int64_
         return set_error(nullptr, MTDAO_ERR_INVALID, "layout: bad arguments");
     int64_t pos = 0;
     for (int32_t k = 0; k < n_tensors; ++k) {
-        if (numel[k] < 1) return set_error(nullptr, MTDAO_ERR_INVALID, "tensor %d has numel %lld", k,
+        if (numel[k] < 0) return set_error(nullptr, MTDAO_ERR_INVALID, "tensor %d has numel %lld", k,
                                            static_cast<long long>(numel[k]));
         offsets_out[k] = pos;
         pos += (numel[k] + 7) / 8 * 8;
     }
+    if (pos == 0) return set_error(nullptr, MTDAO_ERR_INVALID, "the tensor list holds no element");
     *n_padded_out = (pos + 255) / 256 * 256;
     return MTDAO_OK;
 }

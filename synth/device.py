@@ -19,15 +19,23 @@ _lib = None
 
 
 def build(force: bool = False) -> str:
-    if not force and os.path.exists(LIB) and os.path.getmtime(LIB) >= os.path.getmtime(SRC):
+    import fcntl
+
+    def fresh():
+        return os.path.exists(LIB) and os.path.getmtime(LIB) >= os.path.getmtime(SRC)
+
+    if not force and fresh():
         return LIB
     os.makedirs(os.path.dirname(LIB), exist_ok=True)
-    nvcc = shutil.which("nvcc") or "/usr/local/cuda/bin/nvcc"
-    tmp = LIB + ".%d.tmp" % os.getpid()
-    cmd = [nvcc, "-gencode", "arch=compute_103a,code=sm_103a", "-O3", "-std=c++17",
-           "-Xcompiler", "-fPIC", "-shared", SRC, "-o", tmp, "-lcudart"]
-    subprocess.run(cmd, check=True)
-    os.replace(tmp, LIB)
+    with open(os.path.join(os.path.dirname(LIB), ".lock"), "w") as lock:
+        fcntl.flock(lock, fcntl.LOCK_EX)           # one builder at a time
+        if force or not fresh():
+            nvcc = shutil.which("nvcc") or "/usr/local/cuda/bin/nvcc"
+            tmp = LIB + ".%d.tmp" % os.getpid()
+            cmd = [nvcc, "-gencode", "arch=compute_103a,code=sm_103a", "-O3", "-std=c++17",
+                   "-Xcompiler", "-fPIC", "-shared", SRC, "-o", tmp, "-lcudart"]
+            subprocess.run(cmd, check=True)
+            os.replace(tmp, LIB)
     return LIB
 
 
@@ -56,8 +64,11 @@ class DeviceInputs:
         self.seed_grad = int(seed_grad)
         self.seed_init = int(seed_init)
         self.n = int(layout["n_padded"])
-        self.off = torch.tensor(layout["offsets"], dtype=torch.int64, device="cuda")
-        self.num = torch.tensor(layout["numels"], dtype=torch.int64, device="cuda")
+        # zero-size tensors own no element; the device search skips them
+        keep = [(o, k) for o, k in zip(layout["offsets"], layout["numels"]) if k > 0]
+        self.off = torch.tensor([o for o, _ in keep], dtype=torch.int64, device="cuda")
+        self.num = torch.tensor([k for _, k in keep], dtype=torch.int64, device="cuda")
+        self.n_tensors = len(keep)
         self.lib = _load()
 
     def _fill(self, out, bf16, kind, seed, stream_id, M, t, sigma):
@@ -66,7 +77,7 @@ class DeviceInputs:
         rc = self.lib.synth_fill(ctypes.c_void_p(out.data_ptr()), int(bf16), int(kind), seed, stream_id,
                                  M, self.n, int(t), ctypes.c_float(sigma),
                                  ctypes.c_void_p(self.off.data_ptr()), ctypes.c_void_p(self.num.data_ptr()),
-                                 len(self.lay["offsets"]), ctypes.c_void_p(st))
+                                 self.n_tensors, ctypes.c_void_p(st))
         if rc != 0:
             raise RuntimeError("synth_fill failed with CUDA error %d" % rc)
 

@@ -147,8 +147,9 @@ def round_bf16(x: np.ndarray) -> np.ndarray:
 def in_tensor_mask(idx, offsets, numels) -> np.ndarray:
     """True where a padded index lies inside a tensor (not in padding)."""
     idx = np.asarray(idx, np.int64)
-    offsets = np.asarray(offsets, np.int64)
-    numels = np.asarray(numels, np.int64)
+    keep = np.asarray(numels, np.int64) > 0          # zero-size tensors own no index
+    offsets = np.asarray(offsets, np.int64)[keep]
+    numels = np.asarray(numels, np.int64)[keep]
     pos = np.searchsorted(offsets, idx, side="right") - 1
     pos = np.clip(pos, 0, len(offsets) - 1)
     return (idx >= offsets[pos]) & (idx < offsets[pos] + numels[pos])

@@ -41,7 +41,7 @@ def decoder_shapes(vocab: int, d: int, ffn: int, blocks: int) -> list[int]:
 def layout(numels) -> dict:
     """Padded offsets of a flattened multi-tensor list (see module doc)."""
     offsets, pos = [], 0
-    for k in numels:
+    for k in numels:                       # zero-size tensors take no space
         offsets.append(pos)
         pos += (int(k) + TENSOR_ALIGN - 1) // TENSOR_ALIGN * TENSOR_ALIGN
     n_padded = (pos + SLAB_ALIGN - 1) // SLAB_ALIGN * SLAB_ALIGN

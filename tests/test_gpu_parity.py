@@ -339,3 +339,43 @@ def test_device_generator_matches_host_generator(P):
             assert np.array_equal(got.view(np.uint32), expect.view(np.uint32)), name
         x0 = dev.init_params().cpu().numpy()[idx]
         assert np.array_equal(x0, G.init_params(w, lay, SEED_I, idx))
+
+
+def test_zero_size_and_single_element_tensors(P):
+    for shapes in ([0, 5, 0, 300, 0], [1]):
+        w = workload_dict(shapes, 2, betas=(0.9, 0.999), px=2, pu=3, pv=2)
+        eng = gpu_run(P, w, 7)
+        lay = W.layout(w["shapes"])
+        ref = oracle_run(w["opt"], 2, np.arange(lay["n_padded"]), 7, lay, w, SEED_G, SEED_I)
+        compare(gpu_states(eng, w["opt"]), ref)
+        eng.close()
+
+
+@pytest.mark.parametrize("case", ["qhm_beta0_no_grad_term", "omega0", "sgdm_sum_omega1",
+                                  "adopt_beta0", "max_replicas"])
+def test_degenerate_hyperparameters(P, case):
+    M, base, betas, om, kw = 4, "adam", (0.0, 0.999), (0.5, 0.5), {}
+    if case == "omega0":
+        betas, om = (0.9, 0.99), (0.0, 0.0)
+    elif case == "sgdm_sum_omega1":
+        base, betas, om = "sgdm", (0.5, 0.99), (0.3, 0.7)
+    elif case == "adopt_beta0":
+        base, betas, om, kw = "adopt", (0.0, 0.9), (0.5, 0.25), {"beta2": 0.9999, "lr": 2.0 ** -8}
+    elif case == "max_replicas":
+        M, betas, om = P.MAX_REPLICAS, (0.9,), (0.95,)
+    w = workload_dict([3000, 17], M, base=base, betas=betas, omega=om, px=3, pu=2, pv=3, **kw)
+    eng = gpu_run(P, w, 8)
+    lay = W.layout(w["shapes"])
+    ref = oracle_run(w["opt"], M, np.arange(lay["n_padded"]), 8, lay, w, SEED_G, SEED_I)
+    compare(gpu_states(eng, w["opt"]), ref)
+    eng.close()
+
+
+def test_zero_learning_rate_leaves_parameters_bitwise(P):
+    w = workload_dict(RAGGED, 4, betas=(0.9, 0.999), px=0, pu=3, pv=3)
+    lay = W.layout(w["shapes"])
+    x0 = G.init_params(w, lay, SEED_I, np.arange(lay["n_padded"]))
+    eng = gpu_run(P, w, 6, lr=0.0, x0=x0)
+    got = eng.state_view(0).cpu().numpy()
+    assert np.array_equal(got.view(np.uint32), np.tile(x0, (4, 1)).view(np.uint32))
+    eng.close()
