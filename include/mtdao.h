@@ -46,7 +46,7 @@ extern "C" {
 
 #define MTDAO_VERSION 2
 #define MTDAO_MAX_MOM 4          /* largest N supported */
-#define MTDAO_MAX_REPLICAS 64    /* largest M supported */
+#define MTDAO_MAX_REPLICAS 1024  /* largest M supported */
 
 typedef enum {
     MTDAO_OK = 0,
@@ -224,8 +224,10 @@ int mtdao_step_host(mtdao_handle h, const void *grads_host, int32_t grad_dtype, 
 /*
  * Outer synchronisation (Algorithms 1-3, E_m[.] with OuterOpt = averaging):
  * every state in mask is replaced, on every replica, by the equal-weight
- * mean over the M replicas.  Computed as s_0 + (sum_m (s_m - s_0)) / M in
- * fp32, which returns s_0 exactly when the replicas agree.  mask 0 is a no-op.
+ * mean over the M replicas.  Computed in fp32 as s_0 + S / M with S the
+ * Kahan-compensated sum of (s_m - s_0) in replica order, which returns s_0
+ * bit for bit when the replicas agree; the fused average in mtdao_step and
+ * mtdao_sync_stats use the same routine.  mask 0 is a no-op.
  */
 int mtdao_sync(mtdao_handle h, uint32_t mask);
 

@@ -18,7 +18,7 @@ import os
 from .build import LIB as _LIB_PATH
 
 MAX_MOM = 4
-MAX_REPLICAS = 64
+MAX_REPLICAS = 1024
 
 OK, ERR_INVALID, ERR_OOM, ERR_CUDA, ERR_ALIGN, ERR_STATE = 0, -1, -2, -3, -4, -5
 BASE_ADAM, BASE_ADOPT, BASE_SGDM = 0, 1, 2

@@ -3,7 +3,7 @@
 //
 // Averaging (Algorithms 1-3, E_m[.] with averaging as OuterOpt): for every
 // selected state and element, the M replica values are read once and the
-// mean is written back to all M replicas.  Algorithmic traffic: 8 * M bytes
+// mean (replica_mean.cuh) is written back to all M replicas.  Algorithmic traffic: 8 * M bytes
 // per element per state.  HBM-bound; grid-stride over float4 vectors, one
 // grid row (blockIdx.y) per selected state.
 //
@@ -16,6 +16,7 @@
 #include <cstdint>
 
 #include "mtdao_internal.h"
+#include "replica_mean.cuh"
 #include "step_kernels.cuh"
 
 namespace mtdao {
@@ -32,8 +33,10 @@ __global__ void __launch_bounds__(kThreads) sync_kernel(const SyncArgs a) {
     for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < nv;
          i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
         const int64_t e = 4 * i;
-        float s0[4], d[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+        float s0[4];
         to_array(ld_state(base + e), s0);
+        ReplicaMean acc[4] = {ReplicaMean(s0[0]), ReplicaMean(s0[1]), ReplicaMean(s0[2]),
+                              ReplicaMean(s0[3])};
         if constexpr (MT > 0) {
             float r[MT][4];
 #pragma unroll
@@ -41,18 +44,18 @@ __global__ void __launch_bounds__(kThreads) sync_kernel(const SyncArgs a) {
 #pragma unroll
             for (int m = 1; m < MT; ++m)
 #pragma unroll
-                for (int k = 0; k < 4; ++k) d[k] += r[m][k] - s0[k];
+                for (int k = 0; k < 4; ++k) acc[k].add(r[m][k]);
         } else {
             for (int m = 1; m < M; ++m) {
                 float r[4];
                 to_array(ld_state(base + m * n + e), r);
 #pragma unroll
-                for (int k = 0; k < 4; ++k) d[k] += r[k] - s0[k];
+                for (int k = 0; k < 4; ++k) acc[k].add(r[k]);
             }
         }
         float mean[4];
 #pragma unroll
-        for (int k = 0; k < 4; ++k) mean[k] = s0[k] + d[k] / Mf;
+        for (int k = 0; k < 4; ++k) mean[k] = acc[k].value(Mf);
         const float4 mv = from_array(mean);
         for (int m = 0; m < M; ++m) st_state(base + m * n + e, mv);
     }
@@ -167,10 +170,10 @@ __global__ void __launch_bounds__(kThreads) sync_stats_kernel(const SyncArgs a, 
         float mean[4];
 #pragma unroll
         for (int k = 0; k < 4; ++k) {
-            float d = 0.0f;
+            ReplicaMean acc(r[0][k]);
 #pragma unroll
-            for (int m = 1; m < M; ++m) d += r[m][k] - r[0][k];
-            mean[k] = r[0][k] + d / static_cast<float>(M);
+            for (int m = 1; m < M; ++m) acc.add(r[m][k]);
+            mean[k] = acc.value(static_cast<float>(M));
         }
         float q[Q];
 #pragma unroll

@@ -7,6 +7,7 @@
 // average costs no HBM traffic beyond the step's own.
 #pragma once
 
+#include "replica_mean.cuh"
 #include "step_kernels.cuh"
 
 namespace mtdao {
@@ -54,10 +55,9 @@ template <int M>
 __host__ __device__ constexpr int sync_lane_width() { return M <= 4 ? 4 : 2; }
 
 // Writes the M replicas' values of one state for V elements: either as they
-// are, or (when the state is due) all M replaced by the replica mean
-// s_0 + (sum_{m>=1} (s_m - s_0)) / M, summed in replica order.  The
-// standalone averaging kernel uses the same expression and order, so fused
-// and separate averaging give identical bits.
+// are, or (when the state is due) all M replaced by the replica mean of
+// replica_mean.cuh.  The standalone averaging kernels use the same routine,
+// so fused and separate averaging give identical bits.
 template <int M, int V>
 __device__ __forceinline__ void store_replicas(float *state, int64_t n_padded, int64_t e,
                                                float (&val)[M][V], bool average) {
@@ -65,10 +65,10 @@ __device__ __forceinline__ void store_replicas(float *state, int64_t n_padded, i
         float mean[V];
 #pragma unroll
         for (int k = 0; k < V; ++k) {
-            float d = 0.0f;
+            ReplicaMean acc(val[0][k]);
 #pragma unroll
-            for (int m = 1; m < M; ++m) d += val[m][k] - val[0][k];
-            mean[k] = val[0][k] + d / static_cast<float>(M);
+            for (int m = 1; m < M; ++m) acc.add(val[m][k]);
+            mean[k] = acc.value(static_cast<float>(M));
         }
 #pragma unroll
         for (int m = 0; m < M; ++m) st_state_v<V>(state + m * n_padded + e, mean);

@@ -50,6 +50,10 @@ def _load():
                                    ctypes.c_uint64, ctypes.c_int, ctypes.c_int64, ctypes.c_int64,
                                    ctypes.c_float, ctypes.c_void_p, ctypes.c_void_p, ctypes.c_int,
                                    ctypes.c_void_p]
+        lib.synth_toy_grad.restype = ctypes.c_int
+        lib.synth_toy_grad.argtypes = [ctypes.c_int, ctypes.c_void_p, ctypes.c_void_p, ctypes.c_int,
+                                       ctypes.c_int64, ctypes.c_int64, ctypes.c_uint64, ctypes.c_int64,
+                                       ctypes.c_float, ctypes.c_void_p, ctypes.c_void_p]
         _lib = lib
     return _lib
 
@@ -99,3 +103,20 @@ class DeviceInputs:
             out = torch.empty((self.n,), dtype=torch.float32, device="cuda")
         self._fill(out, False, 0, self.seed_init, 2, 1, 0, float(self.w.get("init_sigma", 0.02)))
         return out
+
+
+TOY_KINDS = {"quadratic": 0, "rosenbrock": 1}
+
+
+def toy_grad(kind: str, x_ptr: int, g, M: int, n_padded: int, n_real: int, seed: int, t: int,
+             sigma: float, lam=None) -> None:
+    """Noisy toy-objective gradient of the workers' parameters at device
+    pointer x_ptr ([M][n_padded] fp32) into the float32 tensor g."""
+    import torch
+    lib = _load()
+    st = torch.cuda.current_stream().cuda_stream
+    rc = lib.synth_toy_grad(TOY_KINDS[kind], ctypes.c_void_p(x_ptr), ctypes.c_void_p(g.data_ptr()), M,
+                            n_padded, n_real, seed, int(t), ctypes.c_float(sigma),
+                            ctypes.c_void_p(lam.data_ptr() if lam is not None else 0), ctypes.c_void_p(st))
+    if rc != 0:
+        raise RuntimeError("synth_toy_grad failed with CUDA error %d" % rc)

@@ -170,3 +170,36 @@ def init_params(workload: dict, layout: dict, seed: int, idx) -> np.ndarray:
     x = init_values(seed, idx, workload.get("init_sigma", 0.02))
     inside = in_tensor_mask(idx, layout["offsets"], layout["numels"])
     return np.where(inside, x, np.float32(0.0)).astype(np.float32)
+
+
+STREAM_TOY_NOISE = 3
+
+
+def toy_noise(seed: int, m: int, t: int, idx) -> np.ndarray:
+    """Standard normal noise of the toy objectives (stream 3), float32."""
+    return normal(element_hash(key(seed, STREAM_TOY_NOISE, m, t), idx), 0)
+
+
+def toy_grad(kind: str, x: np.ndarray, seed: int, t: int, sigma: float, lam=None,
+             idx=None) -> np.ndarray:
+    """Noisy gradient of a toy objective at the workers' parameters x
+    ([M][n], any float type; computed in fp64):
+      quadratic   f = sum_i lam_i x_i^2 / 2            g_i = lam_i x_i
+      rosenbrock  f = sum_k (1-a_k)^2 + 100 (b_k - a_k^2)^2 over the pairs
+                  (a_k, b_k) = (x_2k, x_2k+1)
+    plus sigma * Z with Z from stream 3 at padded indices idx (default
+    0..n-1; for Rosenbrock idx must hold whole pairs in order)."""
+    x = np.asarray(x, np.float64)
+    M, n = x.shape
+    idx = np.arange(n) if idx is None else np.asarray(idx, np.int64)
+    if kind == "quadratic":
+        g = np.asarray(lam, np.float64)[None, :] * x
+    elif kind == "rosenbrock":
+        a, b = x[:, 0::2], x[:, 1::2]
+        g = np.empty_like(x)
+        g[:, 0::2] = 2.0 * (a - 1.0) - 400.0 * a * (b - a * a)
+        g[:, 1::2] = 200.0 * (b - a * a)
+    else:
+        raise ValueError(kind)
+    noise = np.stack([toy_noise(seed, m, t, idx) for m in range(M)]).astype(np.float64)
+    return g + float(np.float32(sigma)) * noise

@@ -91,7 +91,61 @@ __global__ void fill_kernel(void *out, int bf16, int kind, uint64_t seed, uint64
     }
 }
 
+// Gradient of a toy objective at each worker's current parameters, plus
+// noise sigma * Z (Z from stream 3: key(seed, 3, m, t), element i, word 0).
+//   kind 0, quadratic  f = sum_i lambda_i x_i^2 / 2:   g_i = lambda_i x_i
+//   kind 1, Rosenbrock f = sum_k (1 - a_k)^2 + 100 (b_k - a_k^2)^2 over the
+//           pairs (a_k, b_k) = (x_2k, x_2k+1):
+//           g_a = 2 (a - 1) - 400 a (b - a^2),   g_b = 200 (b - a^2)
+// Elements at or beyond n_real are padding and get 0.
+__global__ void toy_grad_kernel(int kind, const float *x, float *g, int M, int64_t n, int64_t n_real,
+                                uint64_t seed, int64_t t, float sigma, const float *lam) {
+    const int64_t total = static_cast<int64_t>(M) * n;
+    for (int64_t f = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; f < total;
+         f += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+        const int64_t m = f / n, i = f - m * n;
+        float out = 0.0f;
+        if (i < n_real) {
+            const uint64_t key = mix(mix(mix(seed ^ 3ull) ^ static_cast<uint64_t>(m)) ^
+                                     static_cast<uint64_t>(t));
+            const float z = irwin_hall_normal(mix(key ^ static_cast<uint64_t>(i)), 0);
+            // evaluated in double (toy sizes make that free) so that the
+            // objective's own rounding -- b - a^2 cancels near the valley --
+            // stays far below the optimizer's
+            double grad;
+            if (kind == 0) {
+                grad = static_cast<double>(lam[i]) * static_cast<double>(x[f]);
+            } else {
+                const int64_t base = f - (i & 1);
+                const double a = x[base], b = x[base + 1];
+                const double r = b - a * a;
+                grad = (i & 1) ? 200.0 * r : 2.0 * (a - 1.0) - 400.0 * a * r;
+            }
+            out = static_cast<float>(grad + static_cast<double>(sigma) * static_cast<double>(z));
+        }
+        g[f] = out;
+    }
+}
+
 }  // namespace
+
+// Toy-objective gradients for the M workers' parameters x_dev ([M][n_padded]
+// fp32, e.g. state 0 of an MT-DAO handle) into g_dev ([M][n_padded] fp32).
+// kind 0: quadratic with per-element curvature lam_dev ([n_padded]);
+// kind 1: Rosenbrock pairs (n_real even).  Returns a cudaError_t value.
+extern "C" int synth_toy_grad(int kind, const float *x_dev, float *g_dev, int M, int64_t n_padded,
+                              int64_t n_real, uint64_t seed, int64_t t, float sigma,
+                              const float *lam_dev, void *cuda_stream) {
+    if (x_dev == nullptr || g_dev == nullptr || M < 1 || n_padded < 1 || n_real > n_padded ||
+        (kind == 0 && lam_dev == nullptr) || (kind == 1 && (n_real & 1)) || kind < 0 || kind > 1)
+        return cudaErrorInvalidValue;
+    const int64_t total = static_cast<int64_t>(M) * n_padded;
+    int64_t grid = (total + 255) / 256;
+    if (grid > 4096) grid = 4096;
+    toy_grad_kernel<<<static_cast<unsigned>(grid), 256, 0, static_cast<cudaStream_t>(cuda_stream)>>>(
+        kind, x_dev, g_dev, M, n_padded, n_real, seed, t, sigma, lam_dev);
+    return static_cast<int>(cudaGetLastError());
+}
 
 // Fill out_dev[M][n_padded] (f32, or bf16 when bf16 != 0) for step t.
 // kind: 0 normal, 1 student_t3, 2 normal_outliers.  stream_id: 1 gradients,

@@ -118,7 +118,7 @@ def test_valid_configurations(P):
     with pytest.raises(P.MTDAOError):
         P.mtdao_config_validate(P.make_config(_opt()), 0)
     with pytest.raises(P.MTDAOError):
-        P.mtdao_config_validate(P.make_config(_opt()), 65)
+        P.mtdao_config_validate(P.make_config(_opt()), P.MAX_REPLICAS + 1)
 
 
 def test_null_handle_is_safe(P):

@@ -363,7 +363,8 @@ def test_degenerate_hyperparameters(P, case):
         base, betas, om, kw = "adopt", (0.0, 0.9), (0.5, 0.25), {"beta2": 0.9999, "lr": 2.0 ** -8}
     elif case == "max_replicas":
         M, betas, om = P.MAX_REPLICAS, (0.9,), (0.95,)
-    w = workload_dict([3000, 17], M, base=base, betas=betas, omega=om, px=3, pu=2, pv=3, **kw)
+    shapes = [300, 5] if case == "max_replicas" else [3000, 17]
+    w = workload_dict(shapes, M, base=base, betas=betas, omega=om, px=3, pu=2, pv=3, **kw)
     eng = gpu_run(P, w, 8)
     lay = W.layout(w["shapes"])
     ref = oracle_run(w["opt"], M, np.arange(lay["n_padded"]), 8, lay, w, SEED_G, SEED_I)

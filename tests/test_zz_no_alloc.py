@@ -65,8 +65,8 @@ def test_static_scratch_norm_matches_handle_version():
         eng.close()
 
     w, n, _, g = _grads([1024], 2, "f32", 1.0, 13)
-    out = torch.zeros(65, dtype=torch.float64, device="cuda")
-    for M, npad in ((65, n), (0, n), (2, 100)):
+    out = torch.zeros(8, dtype=torch.float64, device="cuda")
+    for M, npad in ((P.MAX_REPLICAS + 1, n), (0, n), (2, 100)):
         with pytest.raises(P.MTDAOError) as e:
             P.mtdao_grad_sqnorm_static(g.data_ptr(), P.F32, M, npad, out.data_ptr(), stream)
         assert e.value.code == P.ERR_INVALID
