@@ -77,10 +77,18 @@ def source_sha() -> str:
         return hashlib.sha256(f.read()).hexdigest()[:16]
 
 
-def measured_traffic(workload: str, per_launch_units: int):
+def step_kernel_name(opt: dict, grad_dtype: str) -> str:
+    """Template instance of the plain step kernel a workload launches."""
+    base = {"adam": 0, "adopt": 1, "sgdm": 2}[opt["base"]]
+    clip = 1 if opt.get("clip_mode") == "global_norm" else 0
+    return "step_kernel<%d, %d, %d, %d>" % (base, opt["n_mom"], 1 if grad_dtype == "bf16" else 0, clip)
+
+
+def measured_traffic(kernel: str, per_launch_units: int):
     """DRAM bytes per launch of the step kernel from the committed ncu
-    summary, scaled by elements to this launch; None if absent or if the
-    kernel source changed since the capture."""
+    summary, scaled by elements to this launch; None if absent, if it was
+    taken on another template instance, or if the kernel source changed
+    since the capture."""
     rec = {}
     try:
         with open(TRAFFIC_FILE) as f:
@@ -89,7 +97,7 @@ def measured_traffic(workload: str, per_launch_units: int):
                 if line and not line.startswith("#") and "=" in line:
                     k, v = line.split("=", 1)
                     rec[k] = v
-        if rec.get("source_sha") != source_sha():
+        if rec.get("source_sha") != source_sha() or rec.get("kernel") != kernel:
             return None
         per_unit = float(rec["dram_bytes"]) / float(rec["elements"])
     except Exception:
@@ -384,7 +392,7 @@ def run_ours(args):
         cpu = {"value": rate, "unit": "params/s", "cores": 1, "kind": "oracle", "sample": desc,
                "seconds": round(spent, 2)}
 
-    traffic = measured_traffic(w["name"], M * n)
+    traffic = measured_traffic(step_kernel_name(opt, w["grad_dtype"]), M * n)
     line = {
         "metric": "fused MT-DAO step params/s (replica-parameter updates per second, syncs included)",
         "value": value,
@@ -420,7 +428,7 @@ def run_ours(args):
                               if stats_ms else None),
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                      "frac": achieved / peak, "traffic": traffic, "peak_kind": peak_kind,
-                     "kernel": "step_kernel (local step, no sync)"},
+                     "kernel": step_kernel_name(opt, w["grad_dtype"])},
         "cpu_baseline": cpu,
         "e2e": e2e,
         "gpu_launches": args.steps * H * (3 if opt.get("clip_mode") == "global_norm" else 1),
