@@ -33,29 +33,32 @@ __global__ void __launch_bounds__(kThreads) sync_kernel(const SyncArgs a) {
     for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < nv;
          i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
         const int64_t e = 4 * i;
-        float s0[4];
-        to_array(ld_state(base + e), s0);
-        ReplicaMean acc[4] = {ReplicaMean(s0[0]), ReplicaMean(s0[1]), ReplicaMean(s0[2]),
-                              ReplicaMean(s0[3])};
+        float mean[4];
         if constexpr (MT > 0) {
             float r[MT][4];
 #pragma unroll
-            for (int m = 1; m < MT; ++m) to_array(ld_state(base + m * n + e), r[m]);
+            for (int m = 0; m < MT; ++m) to_array(ld_state(base + m * n + e), r[m]);
 #pragma unroll
-            for (int m = 1; m < MT; ++m)
-#pragma unroll
-                for (int k = 0; k < 4; ++k) acc[k].add(r[m][k]);
+            for (int k = 0; k < 4; ++k) mean[k] = replica_mean<MT>([&](int m) { return r[m][k]; });
         } else {
+            // streamed: replicas 1 .. h-1 feed part A, h .. M-1 part B (replica_mean.cuh)
+            float s0[4];
+            to_array(ld_state(base + e), s0);
+            DiffSum pa[4] = {DiffSum(s0[0]), DiffSum(s0[1]), DiffSum(s0[2]), DiffSum(s0[3])};
+            DiffSum pb[4] = {DiffSum(s0[0]), DiffSum(s0[1]), DiffSum(s0[2]), DiffSum(s0[3])};
+            const int h = M / 2;
             for (int m = 1; m < M; ++m) {
                 float r[4];
                 to_array(ld_state(base + m * n + e), r);
 #pragma unroll
-                for (int k = 0; k < 4; ++k) acc[k].add(r[k]);
+                for (int k = 0; k < 4; ++k) {
+                    if (m < h) pa[k].add(r[k]);
+                    else pb[k].add(r[k]);
+                }
             }
-        }
-        float mean[4];
 #pragma unroll
-        for (int k = 0; k < 4; ++k) mean[k] = acc[k].value(Mf);
+            for (int k = 0; k < 4; ++k) mean[k] = replica_mean_from_parts(s0[k], pa[k].partial(), pb[k].partial(), Mf);
+        }
         const float4 mv = from_array(mean);
         for (int m = 0; m < M; ++m) st_state(base + m * n + e, mv);
     }
@@ -169,12 +172,7 @@ __global__ void __launch_bounds__(kThreads) sync_stats_kernel(const SyncArgs a, 
         for (int m = 0; m < M; ++m) to_array(ld_state(base + m * n + e), r[m]);
         float mean[4];
 #pragma unroll
-        for (int k = 0; k < 4; ++k) {
-            ReplicaMean acc(r[0][k]);
-#pragma unroll
-            for (int m = 1; m < M; ++m) acc.add(r[m][k]);
-            mean[k] = acc.value(static_cast<float>(M));
-        }
+        for (int k = 0; k < 4; ++k) mean[k] = replica_mean<M>([&](int m) { return r[m][k]; });
         float q[Q];
 #pragma unroll
         for (int j = 0; j < Q; ++j) q[j] = 0.0f;

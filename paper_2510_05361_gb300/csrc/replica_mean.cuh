@@ -2,24 +2,28 @@
 // every kernel that averages (fused step + sync, sync, sync + diagnostics),
 // so that all of them produce the same bits.
 //
-// mean = s_0 + S / M, where S is the Kahan-compensated sum of (s_m - s_0)
-// over m = 1..M-1 in replica order.  Summing differences keeps the operands
-// small when the replicas are close (the usual case between syncs); the
-// compensation keeps the error of S near one rounding instead of growing
-// with M (a plain fp32 running sum loses about M ulps relative to a mean that
-// is small against the replicas, e.g. 1e-4 at M = 1024).  When S is zero --
-// in particular when all replicas agree -- the result is s_0 itself, bit for
-// bit (sign of zero included).
+// With h = floor(M / 2):
+//   A = Kahan-compensated sum of (s_m - s_0), m = 1 .. h-1, in replica order
+//   B = Kahan-compensated sum of (s_m - s_0), m = h .. M-1, in replica order
+//   mean = s_0 + (A + B) / M      (s_0 itself, bit for bit, when A + B = 0)
+// Summing differences keeps the operands small when the replicas are close
+// (the usual case between syncs); the compensation keeps the error near one
+// rounding instead of growing with M (a plain fp32 running sum loses about M
+// ulps relative to a mean that is small against the replicas, 1e-4 at
+// M = 1024).  The two parts let a kernel hold the replicas of one element
+// in two lanes (replicas 0 .. h-1 and h .. M-1) and still produce exactly
+// the value a single thread computes.
 #pragma once
 
 #include <cuda_runtime.h>
 
 namespace mtdao {
 
-struct ReplicaMean {
+// Kahan-compensated sum of differences to a reference value s0.
+struct DiffSum {
     float s0, sum, comp;
 
-    __device__ __forceinline__ explicit ReplicaMean(float first) : s0(first), sum(0.0f), comp(0.0f) {}
+    __device__ __forceinline__ explicit DiffSum(float ref) : s0(ref), sum(0.0f), comp(0.0f) {}
 
     __device__ __forceinline__ void add(float sm) {
         const float y = (sm - s0) - comp;
@@ -28,10 +32,36 @@ struct ReplicaMean {
         sum = t;
     }
 
-    __device__ __forceinline__ float value(float M) const {
-        const float q = (sum - comp) / M;
-        return q == 0.0f ? s0 : s0 + q;
-    }
+    __device__ __forceinline__ float partial() const { return sum - comp; }
 };
+
+__device__ __forceinline__ float replica_mean_from_parts(float s0, float part_a, float part_b, float M) {
+    const float q = (part_a + part_b) / M;
+    return q == 0.0f ? s0 : s0 + q;
+}
+
+// The mean of M values held by one thread; get(m) returns replica m's value.
+template <int M, typename Get>
+__device__ __forceinline__ float replica_mean(Get get) {
+    constexpr int h = M / 2;
+    const float s0 = get(0);
+    DiffSum a(s0), b(s0);
+#pragma unroll
+    for (int m = 1; m < h; ++m) a.add(get(m));
+#pragma unroll
+    for (int m = (h > 1 ? h : 1); m < M; ++m) b.add(get(m));
+    return replica_mean_from_parts(s0, a.partial(), b.partial(), static_cast<float>(M));
+}
+
+// Same, for a replica count known only at run time.
+template <typename Get>
+__device__ __forceinline__ float replica_mean_rt(int M, Get get) {
+    const int h = M / 2;
+    const float s0 = get(0);
+    DiffSum a(s0), b(s0);
+    for (int m = 1; m < h; ++m) a.add(get(m));
+    for (int m = (h > 1 ? h : 1); m < M; ++m) b.add(get(m));
+    return replica_mean_from_parts(s0, a.partial(), b.partial(), static_cast<float>(M));
+}
 
 }  // namespace mtdao

@@ -1,10 +1,11 @@
 // step_sync_kernels.cuh -- the local step with the replica average fused in.
 //
-// step_sync_kernel is element-major: a lane updates the same V elements
-// (V = 4 for M <= 4, V = 2 for M = 8) of all M replicas with the update of
-// step_kernels.cuh, then writes each state due for averaging as the replica
-// mean (E_m[.] of Algorithms 1-3) instead of the M local values.  The
-// average costs no HBM traffic beyond the step's own.
+// step_sync_kernel is element-major: a lane updates the same 4 elements of
+// all M replicas (M <= 4) or, for M = 8, of 4 replicas while the lane 16
+// places away holds the other 4, with the update of step_kernels.cuh; then
+// it writes each state due for averaging as the replica mean (E_m[.] of
+// Algorithms 1-3) instead of the local values.  The average costs no HBM
+// traffic beyond the step's own.
 #pragma once
 
 #include "replica_mean.cuh"
@@ -14,19 +15,40 @@ namespace mtdao {
 
 // ---------------------------------------------------------------- fused step + sync
 
-// V consecutive fp32 states (V = 4: one 128-bit access, V = 2: one 64-bit
-// access) and V gradient elements, upcast to fp32.
+// Layout of the fused kernel's work.  A lane holds its elements of R
+// replicas for every state it touches, so registers grow with R * V:
+//   M = 2 : one lane group, R = 2, V = 4 elements (128-bit accesses); the
+//           states are loaded, updated and stored one after another.
+//   M = 4 : one lane group, R = 4, V = 2 (64-bit accesses); every load of
+//           the chunk is issued before any arithmetic, as in step_kernel.
+//   M = 8 : two lane groups (half-warps), R = 4, V = 4, state by state;
+//           lanes q and q + 16 hold the same elements, replicas 0..3 and
+//           4..7, and combine their parts of the average by shuffles.
+// Measured on the flat 2^27 sweep (GB/s of the fused step, Adam, f32):
+// issuing all loads first lifts M = 4 from ~6180 to ~6480 (the plain step's
+// level) but costs M = 2 (6650 -> 6500) and M = 8 (5840 -> 5000-5760,
+// register spills), hence the split.
+template <int M>
+struct FusedShape {
+    static constexpr int G = M == 8 ? 2 : 1;      // lane groups per warp
+    static constexpr int R = M / G;               // replicas per lane
+    static constexpr bool kPrefetch = M == 4;     // all loads of a chunk first
+    static constexpr int V = kPrefetch ? 2 : 4;   // elements per lane
+    static constexpr int kLanes = 32 / G;         // lanes per group
+    static constexpr int kChunk = kLanes * V;     // elements per warp iteration
+};
+
 template <int V>
-__device__ __forceinline__ void ld_state_v(const float *p, float *a) {
+__device__ __forceinline__ void ld_v(const float *p, float *a) {
     if constexpr (V == 4) {
         to_array(ld_state(p), a);
     } else {
-        const float2 v = __ldcs(reinterpret_cast<const float2 *>(p));
-        a[0] = v.x; a[1] = v.y;
+        const float2 t = __ldcs(reinterpret_cast<const float2 *>(p));
+        a[0] = t.x; a[1] = t.y;
     }
 }
 template <int V>
-__device__ __forceinline__ void st_state_v(float *p, const float *a) {
+__device__ __forceinline__ void st_v(float *p, const float *a) {
     if constexpr (V == 4) {
         st_state(p, from_array(a));
     } else {
@@ -38,8 +60,8 @@ __device__ __forceinline__ void ld_grad_v(const void *g, int64_t e, float *a) {
     if constexpr (V == 4) {
         to_array(ld_grad<GDT>(g, e), a);
     } else if constexpr (GDT == MTDAO_F32) {
-        const float2 v = __ldcs(reinterpret_cast<const float2 *>(static_cast<const float *>(g) + e));
-        a[0] = v.x; a[1] = v.y;
+        const float2 t = __ldcs(reinterpret_cast<const float2 *>(static_cast<const float *>(g) + e));
+        a[0] = t.x; a[1] = t.y;
     } else {
         const unsigned int w =
             __ldcs(reinterpret_cast<const unsigned int *>(static_cast<const uint16_t *>(g) + e));
@@ -47,158 +69,201 @@ __device__ __forceinline__ void ld_grad_v(const void *g, int64_t e, float *a) {
     }
 }
 
-// Elements per lane in the fused step+sync kernel: a lane holds its
-// elements of all M replicas for every state it touches, so wide lanes cost
-// registers in proportion to M.  Four elements (128-bit accesses) up to M = 4,
-// two (64-bit accesses, still whole 32-byte sectors per warp) beyond.
+// Writes one state's R local values (for V elements) to the lane's replicas:
+// as they are, or -- when the state is due -- all replaced by the replica
+// mean of replica_mean.cuh.  With two lane groups each group forms its part
+// of the compensated sum (replicas 1..3 and 4..7 against replica 0's value)
+// and the parts are exchanged, so both groups store exactly the value a
+// single thread would compute.  The standalone averaging kernels use the
+// same routine, so fused and separate averaging give identical bits.
 template <int M>
-__host__ __device__ constexpr int sync_lane_width() { return M <= 4 ? 4 : 2; }
-
-// Writes the M replicas' values of one state for V elements: either as they
-// are, or (when the state is due) all M replaced by the replica mean of
-// replica_mean.cuh.  The standalone averaging kernels use the same routine,
-// so fused and separate averaging give identical bits.
-template <int M, int V>
-__device__ __forceinline__ void store_replicas(float *state, int64_t n_padded, int64_t e,
-                                               float (&val)[M][V], bool average) {
+__device__ __forceinline__ void store_replicas(float *state, int64_t n_padded, int64_t e, int grp,
+                                               float (&val)[FusedShape<M>::R][FusedShape<M>::V],
+                                               bool average) {
+    using S = FusedShape<M>;
     if (average) {
-        float mean[V];
+        float mean[S::V];
 #pragma unroll
-        for (int k = 0; k < V; ++k) {
-            ReplicaMean acc(val[0][k]);
+        for (int k = 0; k < S::V; ++k) {
+            if constexpr (S::G == 1) {
+                mean[k] = replica_mean<M>([&](int m) { return val[m][k]; });
+            } else {
+                // replica 0 lives in group 0: its value is the reference of both parts
+                const float s0 = __shfl_sync(0xffffffffu, val[0][k], threadIdx.x & (S::kLanes - 1));
+                DiffSum part(s0);
 #pragma unroll
-            for (int m = 1; m < M; ++m) acc.add(val[m][k]);
-            mean[k] = acc.value(static_cast<float>(M));
+                for (int r = (grp == 0 ? 1 : 0); r < S::R; ++r) part.add(val[r][k]);
+                const float mine = part.partial();
+                const float other = __shfl_xor_sync(0xffffffffu, mine, S::kLanes);
+                const float a = grp == 0 ? mine : other;          // replicas 1 .. 3
+                const float b = grp == 0 ? other : mine;          // replicas 4 .. 7
+                mean[k] = replica_mean_from_parts(s0, a, b, static_cast<float>(M));
+            }
         }
 #pragma unroll
-        for (int m = 0; m < M; ++m) st_state_v<V>(state + m * n_padded + e, mean);
+        for (int r = 0; r < S::R; ++r)
+            st_v<S::V>(state + (grp * S::R + r) * n_padded + e, mean);
     } else {
 #pragma unroll
-        for (int m = 0; m < M; ++m) st_state_v<V>(state + m * n_padded + e, val[m]);
+        for (int r = 0; r < S::R; ++r)
+            st_v<S::V>(state + (grp * S::R + r) * n_padded + e, val[r]);
     }
 }
 
-template <int M, int V>
-__device__ __forceinline__ void load_replicas(const float *state, int64_t n_padded, int64_t e,
-                                              float (&val)[M][V]) {
+template <int M>
+__device__ __forceinline__ void load_replicas(const float *state, int64_t n_padded, int64_t e, int grp,
+                                              float (&val)[FusedShape<M>::R][FusedShape<M>::V]) {
+    using S = FusedShape<M>;
 #pragma unroll
-    for (int m = 0; m < M; ++m) ld_state_v<V>(state + m * n_padded + e, val[m]);
+    for (int r = 0; r < S::R; ++r) ld_v<S::V>(state + (grp * S::R + r) * n_padded + e, val[r]);
 }
 
 template <int BASE, int N, int GDT, bool CLIP, int M>
 __global__ void __launch_bounds__(kThreads, 2) step_sync_kernel(const StepArgs a) {
-    constexpr int V = sync_lane_width<M>();
-    constexpr int kLaneChunk = 32 * V;              // elements per warp iteration
+    using S = FusedShape<M>;
+    constexpr int R = S::R;
+    constexpr int V = S::V;
     const int lane = threadIdx.x & 31;
+    const int q = lane & (S::kLanes - 1);
+    const int grp = lane / S::kLanes;
     const int64_t n = a.n_padded;
-    const int64_t n_chunks = n / kLaneChunk;
+    const int64_t n_chunks = n / S::kChunk;
     const int64_t warp = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
     const int64_t n_warps = (static_cast<int64_t>(gridDim.x) * blockDim.x) >> 5;
     const uint32_t mask = a.sync_mask;
 
-    float s[M];
+    float s[R];
 #pragma unroll
-    for (int m = 0; m < M; ++m) s[m] = CLIP ? __ldg(a.clip_scale + m) : 1.0f;
+    for (int r = 0; r < R; ++r) s[r] = CLIP ? __ldg(a.clip_scale + grp * R + r) : 1.0f;
 
     for (int64_t c = warp; c < n_chunks; c += n_warps) {
-        const int64_t e = c * kLaneChunk + V * lane;
-        float g[M][V];
+        const int64_t e = c * S::kChunk + V * q;
+        float g[R][V];
 #pragma unroll
-        for (int m = 0; m < M; ++m) ld_grad_v<GDT, V>(a.grads, m * n + e, g[m]);
+        for (int r = 0; r < R; ++r) ld_grad_v<GDT, V>(a.grads, (grp * R + r) * n + e, g[r]);
 
-        if constexpr (BASE == MTDAO_BASE_ADOPT) {
+        if constexpr (S::kPrefetch) {
+            // Every load of the chunk is issued before any arithmetic (as in
+            // step_kernel), then the shared per-element update, then the
+            // stores with the due averages.
+            constexpr bool kHasV = BASE != MTDAO_BASE_SGDM;
+            float x[R][V], u[N][R][V], v[R][V];
+            load_replicas<M>(a.arena, n, e, grp, x);
+#pragma unroll
+            for (int j = 0; j < N; ++j) load_replicas<M>(a.arena + (1 + j) * a.stride, n, e, grp, u[j]);
+            if constexpr (kHasV) load_replicas<M>(a.arena + (1 + N) * a.stride, n, e, grp, v);
+#pragma unroll
+            for (int r = 0; r < R; ++r)
+#pragma unroll
+                for (int k = 0; k < V; ++k) {
+                    float uk[N];
+#pragma unroll
+                    for (int j = 0; j < N; ++j) uk[j] = u[j][r][k];
+                    float vk = kHasV ? v[r][k] : 0.0f;
+                    update_element<BASE, N>(a.sc, g[r][k], s[r], x[r][k], uk, vk);
+#pragma unroll
+                    for (int j = 0; j < N; ++j) u[j][r][k] = uk[j];
+                    if constexpr (kHasV) v[r][k] = vk;
+                }
+            store_replicas<M>(a.arena, n, e, grp, x, mask & 1u);
+#pragma unroll
+            for (int j = 0; j < N; ++j)
+                store_replicas<M>(a.arena + (1 + j) * a.stride, n, e, grp, u[j], (mask >> (1 + j)) & 1u);
+            if constexpr (kHasV)
+                store_replicas<M>(a.arena + (1 + N) * a.stride, n, e, grp, v, (mask >> (1 + N)) & 1u);
+        } else if constexpr (BASE == MTDAO_BASE_ADOPT) {
             // v first; g becomes the normalised, clamped gradient.
             {
-                float v[M][V];
+                float v[R][V];
                 float *p = a.arena + (1 + N) * a.stride;
-                load_replicas<M, V>(p, n, e, v);
+                load_replicas<M>(p, n, e, grp, v);
 #pragma unroll
-                for (int m = 0; m < M; ++m)
+                for (int r = 0; r < R; ++r)
 #pragma unroll
                     for (int k = 0; k < V; ++k) {
-                        const float gr = g[m][k];
+                        const float gr = g[r][k];
                         float gn;
                         if (a.sc.prev_v) {
-                            gn = gr / (sqrtf(v[m][k]) + a.sc.eps);
-                            v[m][k] = fmaf(a.sc.c2, fmaf(gr, gr, -v[m][k]), v[m][k]);
+                            gn = gr / (sqrtf(v[r][k]) + a.sc.eps);
+                            v[r][k] = fmaf(a.sc.c2, fmaf(gr, gr, -v[r][k]), v[r][k]);
                         } else {
-                            v[m][k] = fmaf(a.sc.c2, fmaf(gr, gr, -v[m][k]), v[m][k]);
-                            gn = gr / (sqrtf(v[m][k]) + a.sc.eps);
+                            v[r][k] = fmaf(a.sc.c2, fmaf(gr, gr, -v[r][k]), v[r][k]);
+                            gn = gr / (sqrtf(v[r][k]) + a.sc.eps);
                         }
                         gn = gn > a.sc.clip_c ? a.sc.clip_c : (gn < -a.sc.clip_c ? -a.sc.clip_c : gn);
-                        g[m][k] = gn;
+                        g[r][k] = gn;
                     }
-                store_replicas<M, V>(p, n, e, v, (mask >> (1 + N)) & 1u);
+                store_replicas<M>(p, n, e, grp, v, (mask >> (1 + N)) & 1u);
             }
-            float d[M][V];
+            float d[R][V];
 #pragma unroll
-            for (int m = 0; m < M; ++m)
+            for (int r = 0; r < R; ++r)
 #pragma unroll
-                for (int k = 0; k < V; ++k) d[m][k] = a.sc.cg * g[m][k];
+                for (int k = 0; k < V; ++k) d[r][k] = a.sc.cg * g[r][k];
 #pragma unroll
             for (int j = 0; j < N; ++j) {
-                float u[M][V];
+                float u[R][V];
                 float *p = a.arena + (1 + j) * a.stride;
-                load_replicas<M, V>(p, n, e, u);
+                load_replicas<M>(p, n, e, grp, u);
 #pragma unroll
-                for (int m = 0; m < M; ++m)
+                for (int r = 0; r < R; ++r)
 #pragma unroll
                     for (int k = 0; k < V; ++k) {
-                        u[m][k] = fmaf(a.sc.c1[j], g[m][k] - u[m][k], u[m][k]);
-                        d[m][k] = fmaf(a.sc.k[j], u[m][k], d[m][k]);
+                        u[r][k] = fmaf(a.sc.c1[j], g[r][k] - u[r][k], u[r][k]);
+                        d[r][k] = fmaf(a.sc.k[j], u[r][k], d[r][k]);
                     }
-                store_replicas<M, V>(p, n, e, u, (mask >> (1 + j)) & 1u);
+                store_replicas<M>(p, n, e, grp, u, (mask >> (1 + j)) & 1u);
             }
-            float x[M][V];
-            load_replicas<M, V>(a.arena, n, e, x);
+            float x[R][V];
+            load_replicas<M>(a.arena, n, e, grp, x);
 #pragma unroll
-            for (int m = 0; m < M; ++m)
+            for (int r = 0; r < R; ++r)
 #pragma unroll
-                for (int k = 0; k < V; ++k) x[m][k] = fmaf(a.sc.neg_lr, d[m][k], x[m][k]);
-            store_replicas<M, V>(a.arena, n, e, x, mask & 1u);
+                for (int k = 0; k < V; ++k) x[r][k] = fmaf(a.sc.neg_lr, d[r][k], x[r][k]);
+            store_replicas<M>(a.arena, n, e, grp, x, mask & 1u);
         } else {
-            // Adam / SGDM: momenta of the clipped gradient g * s[m], then
+            // Adam / SGDM: momenta of the clipped gradient g * s[r], then
             // (Adam) v of the raw gradient and the denominator, then x.
-            float num[M][V];
+            float num[R][V];
 #pragma unroll
-            for (int m = 0; m < M; ++m)
+            for (int r = 0; r < R; ++r)
 #pragma unroll
-                for (int k = 0; k < V; ++k) num[m][k] = a.sc.cg * __fmul_rn(g[m][k], s[m]);
+                for (int k = 0; k < V; ++k) num[r][k] = a.sc.cg * __fmul_rn(g[r][k], s[r]);
 #pragma unroll
             for (int j = 0; j < N; ++j) {
-                float u[M][V];
+                float u[R][V];
                 float *p = a.arena + (1 + j) * a.stride;
-                load_replicas<M, V>(p, n, e, u);
+                load_replicas<M>(p, n, e, grp, u);
 #pragma unroll
-                for (int m = 0; m < M; ++m)
+                for (int r = 0; r < R; ++r)
 #pragma unroll
                     for (int k = 0; k < V; ++k) {
-                        u[m][k] = fmaf(a.sc.c1[j], __fmul_rn(g[m][k], s[m]) - u[m][k], u[m][k]);
-                        num[m][k] = fmaf(a.sc.k[j], u[m][k], num[m][k]);
+                        u[r][k] = fmaf(a.sc.c1[j], __fmul_rn(g[r][k], s[r]) - u[r][k], u[r][k]);
+                        num[r][k] = fmaf(a.sc.k[j], u[r][k], num[r][k]);
                     }
-                store_replicas<M, V>(p, n, e, u, (mask >> (1 + j)) & 1u);
+                store_replicas<M>(p, n, e, grp, u, (mask >> (1 + j)) & 1u);
             }
             if constexpr (BASE == MTDAO_BASE_ADAM) {
-                float v[M][V];
+                float v[R][V];
                 float *p = a.arena + (1 + N) * a.stride;
-                load_replicas<M, V>(p, n, e, v);
+                load_replicas<M>(p, n, e, grp, v);
 #pragma unroll
-                for (int m = 0; m < M; ++m)
+                for (int r = 0; r < R; ++r)
 #pragma unroll
                     for (int k = 0; k < V; ++k) {
-                        const float gr = g[m][k];
-                        v[m][k] = fmaf(a.sc.c2, fmaf(gr, gr, -v[m][k]), v[m][k]);
-                        num[m][k] = num[m][k] / fmaf(sqrtf(v[m][k]), a.sc.sv, a.sc.eps);
+                        const float gr = g[r][k];
+                        v[r][k] = fmaf(a.sc.c2, fmaf(gr, gr, -v[r][k]), v[r][k]);
+                        num[r][k] = num[r][k] / fmaf(sqrtf(v[r][k]), a.sc.sv, a.sc.eps);
                     }
-                store_replicas<M, V>(p, n, e, v, (mask >> (1 + N)) & 1u);
+                store_replicas<M>(p, n, e, grp, v, (mask >> (1 + N)) & 1u);
             }
-            float x[M][V];
-            load_replicas<M, V>(a.arena, n, e, x);
+            float x[R][V];
+            load_replicas<M>(a.arena, n, e, grp, x);
 #pragma unroll
-            for (int m = 0; m < M; ++m)
+            for (int r = 0; r < R; ++r)
 #pragma unroll
-                for (int k = 0; k < V; ++k) x[m][k] = fmaf(a.sc.neg_lr, num[m][k], x[m][k]);
-            store_replicas<M, V>(a.arena, n, e, x, mask & 1u);
+                for (int k = 0; k < V; ++k) x[r][k] = fmaf(a.sc.neg_lr, num[r][k], x[r][k]);
+            store_replicas<M>(a.arena, n, e, grp, x, mask & 1u);
         }
     }
 }
@@ -209,7 +274,7 @@ template <int BASE, int N, int GDT, bool CLIP, int M>
 cudaError_t launch_step_sync_t(const StepArgs &a, int num_sms, cudaStream_t stream) {
     auto kernel = step_sync_kernel<BASE, N, GDT, CLIP, M>;
     static const int per_sm = blocks_per_sm(kernel);
-    const int grid = persistent_grid(per_sm, num_sms, a.n_padded / (32 * sync_lane_width<M>()));
+    const int grid = persistent_grid(per_sm, num_sms, a.n_padded / FusedShape<M>::kChunk);
     kernel<<<grid, kThreads, 0, stream>>>(a);
     return cudaGetLastError();
 }
