@@ -137,6 +137,20 @@ WORKLOADS = {
         "init_sigma": 0.02,
         "opt": _opt("adam", (0.5, 0.9, 0.999), 0.999, 1e-3, 32, 32, 32),
     },
+    "profile_small_adopt": {
+        "name": "profile_small_adopt",
+        "desc": "flat vector n=2^24 with the ~350M workload's optimizer (M=8, N=2 "
+                "beta=(0.95,0.999), ADOPT beta2=0.9999, bf16 grads N(0,1e-3), H_x=64, "
+                "H_u=H_v=16): the same kernels on ~2.4 GB of device memory, for profiler captures",
+        "shapes": [1 << 24],
+        "M": 8,
+        "T": 64,
+        "grad_kind": "normal",
+        "grad_sigma": 1e-3,
+        "grad_dtype": "bf16",
+        "init_sigma": 0.02,
+        "opt": _opt("adopt", (0.95, 0.999), 0.9999, 2.0 ** -8, 64, 16, 16, bias=False),
+    },
 }
 
 SWEEP_BETAS = (0.9, 0.999, 0.5, 0.99)
