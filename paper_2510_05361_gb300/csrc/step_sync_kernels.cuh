@@ -92,7 +92,8 @@ __device__ __forceinline__ void store_replicas(float *state, int64_t n_padded, i
                 const float s0 = __shfl_sync(0xffffffffu, val[0][k], threadIdx.x & (S::kLanes - 1));
                 DiffSum part(s0);
 #pragma unroll
-                for (int r = (grp == 0 ? 1 : 0); r < S::R; ++r) part.add(val[r][k]);
+                for (int r = 0; r < S::R; ++r)      // constant indices: val stays in registers
+                    if (r > 0 || grp != 0) part.add(val[r][k]);
                 const float mine = part.partial();
                 const float other = __shfl_xor_sync(0xffffffffu, mine, S::kLanes);
                 const float a = grp == 0 ? mine : other;          // replicas 1 .. 3
