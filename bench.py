@@ -360,6 +360,24 @@ def run_ours(args):
             if i >= 2:
                 stats_ms.append(a.elapsed_time(b))
 
+    # pseudo-gradient diagnostics: a read-only pass over x and the anchor
+    pg_ms = []
+    if M <= 8:
+        P.mtdao_track_anchor(eng.h, True)
+        pg_out = torch.empty((2 * M + 2,), dtype=torch.float64, device="cuda")
+        for i in range(6):
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            if flush is not None:
+                flush.fill_(1.0)
+            a.record(stream)
+            P.mtdao_pseudo_grad_stats(eng.h, pg_out.data_ptr())
+            b.record(stream)
+            torch.cuda.synchronize()
+            if i >= 2:
+                pg_ms.append(a.elapsed_time(b))
+        P.mtdao_track_anchor(eng.h, False)
+    pg_bytes = (M + 1) * n * 4
+
     # end to end through the host-buffer C-ABI call
     e2e = None
     if not args.no_e2e and args.e2e_rounds > 0:
@@ -426,6 +444,9 @@ def run_ours(args):
                                "gbs": sync_bytes / (statistics.median(stats_ms) / 1e3) / 1e9,
                                "frac": sync_bytes / (statistics.median(stats_ms) / 1e3) / 1e9 / peak}
                               if stats_ms else None),
+        "pseudo_grad_stats_kernel": ({"ms_median": statistics.median(pg_ms), "bytes": pg_bytes,
+                                      "gbs": pg_bytes / (statistics.median(pg_ms) / 1e3) / 1e9}
+                                     if pg_ms else None),
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                      "frac": achieved / peak, "traffic": traffic, "peak_kind": peak_kind,
                      "kernel": step_kernel_name(opt, w["grad_dtype"])},

@@ -167,6 +167,35 @@ void mto_state_stats(int M, long long n, const double *s, double *out)
     }
 }
 
+/*
+ * Pseudo-gradient diagnostics (section 4.1 "Other Metrics"; section 5.4 uses
+ * the worker update over a round, Delta^m = x^m_{t+K} - x^m_t, and its mean,
+ * the global pseudo-gradient).  a = the parameters at the start of the round
+ * (the last average), x[M][n] the workers' parameters now, x_bar = E_m[x]:
+ *   out[m]           ||x_m - a||^2                         m = 0..M-1
+ *   out[M + m]       <x_m - a, x_bar - a>
+ *   out[2M]          ||x_bar - a||^2
+ *   out[2M + 1]      ||a||^2
+ * so cos(local, global pseudo-gradient) = out[M+m] / sqrt(out[m] out[2M]) and
+ * the relative change of the averaged model = sqrt(out[2M] / out[2M+1]).
+ */
+void mto_pseudo_grad_stats(int M, long long n, const double *x, const double *a, double *out)
+{
+    for (int k = 0; k < 2 * M + 2; ++k) out[k] = 0.0;
+    for (long long i = 0; i < n; ++i) {
+        double sum = 0.0;
+        for (int m = 0; m < M; ++m) sum += x[(long long)m * n + i];
+        double global = sum / (double)M - a[i];
+        out[2 * M] += global * global;
+        out[2 * M + 1] += a[i] * a[i];
+        for (int m = 0; m < M; ++m) {
+            double local = x[(long long)m * n + i] - a[i];
+            out[m] += local * local;
+            out[M + m] += local * global;
+        }
+    }
+}
+
 /* ||g^m||_2 of one worker's flattened gradient, summed in index order. */
 double mto_grad_norm(long long n, const double *g)
 {

@@ -105,6 +105,8 @@ def _load():
             lib.mto_mean_over_workers.restype = None
             lib.mto_state_stats.argtypes = [ctypes.c_int, ctypes.c_longlong, dp, dp]
             lib.mto_state_stats.restype = None
+            lib.mto_pseudo_grad_stats.argtypes = [ctypes.c_int, ctypes.c_longlong, dp, dp, dp]
+            lib.mto_pseudo_grad_stats.restype = None
             _lib = lib
     return _lib
 
@@ -217,6 +219,19 @@ def state_stats(s: np.ndarray) -> np.ndarray:
     M = s.shape[0]
     out = np.zeros(2 + 2 * M, np.float64)
     _load().mto_state_stats(M, s.size // M, _ptr(s), _ptr(out))
+    return out
+
+
+def pseudo_grad_stats(x: np.ndarray, anchor: np.ndarray) -> np.ndarray:
+    """Pseudo-gradient diagnostics of the workers' parameters x ``[M][n]``
+    against the round's starting point ``anchor`` ``[n]`` (see
+    mto_pseudo_grad_stats): [||x_m - a||^2 (M), <x_m - a, x_bar - a> (M),
+    ||x_bar - a||^2, ||a||^2]."""
+    x = np.ascontiguousarray(x, np.float64)
+    a = np.ascontiguousarray(anchor, np.float64).ravel()
+    M = x.shape[0]
+    out = np.zeros(2 * M + 2, np.float64)
+    _load().mto_pseudo_grad_stats(M, a.size, _ptr(x), _ptr(a), _ptr(out))
     return out
 
 

@@ -84,6 +84,8 @@ def _load():
         "mtdao_sync": (ctypes.c_int, [H, ctypes.c_uint32]),
         "mtdao_sync_due": (ctypes.c_int, [H, ctypes.POINTER(ctypes.c_uint32)]),
         "mtdao_sync_stats": (ctypes.c_int, [H, ctypes.c_uint32, ctypes.c_void_p]),
+        "mtdao_track_anchor": (ctypes.c_int, [H, ctypes.c_int32]),
+        "mtdao_pseudo_grad_stats": (ctypes.c_int, [H, ctypes.c_void_p]),
         "mtdao_grad_sqnorm": (ctypes.c_int, [H, ctypes.c_void_p, ctypes.c_int32, ctypes.c_void_p]),
         "mtdao_grad_sqnorm_static": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_int32, ctypes.c_int32,
                                                     ctypes.c_int64, ctypes.c_void_p, ctypes.c_void_p]),
@@ -225,6 +227,14 @@ def mtdao_sync_stats(h, mask: int, stats_dev_ptr: int) -> None:
     _check(lib.mtdao_sync_stats(h, mask, ctypes.c_void_p(stats_dev_ptr)), h)
 
 
+def mtdao_track_anchor(h, enable: bool) -> None:
+    _check(lib.mtdao_track_anchor(h, 1 if enable else 0), h)
+
+
+def mtdao_pseudo_grad_stats(h, out_dev_ptr: int) -> None:
+    _check(lib.mtdao_pseudo_grad_stats(h, ctypes.c_void_p(out_dev_ptr)), h)
+
+
 def mtdao_sync_due(h) -> int:
     m = ctypes.c_uint32()
     _check(lib.mtdao_sync_due(h, ctypes.byref(m)), h)
@@ -351,6 +361,17 @@ class MTDAO:
         k = bin(mask).count("1")
         out = torch.empty((k, 2 + 2 * self.M), dtype=torch.float64, device="cuda")
         mtdao_sync_stats(self.h, mask, out.data_ptr())
+        return out
+
+    def track_anchor(self, enable: bool = True) -> None:
+        mtdao_track_anchor(self.h, enable)
+
+    def pseudo_grad_stats(self):
+        """Pseudo-gradient diagnostics against the anchor as a device tensor
+        [2M + 2] (see mtdao_pseudo_grad_stats)."""
+        import torch
+        out = torch.empty((2 * self.M + 2,), dtype=torch.float64, device="cuda")
+        mtdao_pseudo_grad_stats(self.h, out.data_ptr())
         return out
 
     def state_ptr(self, state: int, replica: int) -> int:

@@ -76,8 +76,9 @@ struct mtdao_ctx {
     double *norm_out = nullptr;       // [M]
     double *norm_partial = nullptr;   // [M][norm_blocks]
     int norm_blocks = 1;
-    double *stats_partial = nullptr;  // mtdao_sync_stats workspace (allocated on first use)
+    double *stats_partial = nullptr;  // diagnostics workspace (allocated on first use)
     size_t stats_cap = 0;
+    float *anchor = nullptr;          // x at the last parameter average (mtdao_track_anchor)
     // host-gradient staging (mtdao_step_host)
     void *staging[2] = {nullptr, nullptr};
     size_t staging_bytes = 0;
@@ -251,6 +252,7 @@ void release(mtdao_ctx *h) {
     if (h->norm_out) cudaFree(h->norm_out);
     if (h->norm_partial) cudaFree(h->norm_partial);
     if (h->stats_partial) cudaFree(h->stats_partial);
+    if (h->anchor) cudaFree(h->anchor);
 }
 
 int check_handle(mtdao_ctx *h) {
@@ -438,6 +440,29 @@ extern "C" int mtdao_set_params(mtdao_handle h, const float *x0_dev) {
 
 // ====================================================================== hot path
 
+// After a step or sync whose mask includes x (bit 0), the tracked anchor
+// becomes the averaged parameters (replica 0's copy).
+static int refresh_anchor(mtdao_ctx *h, uint32_t mask) {
+    if (h->anchor == nullptr || (mask & 1u) == 0) return MTDAO_OK;
+    cudaError_t e = cudaMemcpyAsync(h->anchor, h->arena, static_cast<size_t>(h->n_padded) * sizeof(float),
+                                    cudaMemcpyDeviceToDevice, h->stream);
+    if (e != cudaSuccess) return cuda_fail(h, e, "anchor copy");
+    return MTDAO_OK;
+}
+
+static int ensure_stats_workspace(mtdao_ctx *h) {
+    if (h->stats_partial != nullptr) return MTDAO_OK;
+    const size_t cap = sync_stats_partial_capacity(h->num_sms, h->n_states, h->M);
+    cudaError_t e = cudaMalloc(reinterpret_cast<void **>(&h->stats_partial), cap * sizeof(double));
+    if (e != cudaSuccess) {
+        cudaGetLastError();
+        h->stats_partial = nullptr;
+        return set_error(h, MTDAO_ERR_OOM, "diagnostics workspace: %s", cudaGetErrorString(e));
+    }
+    h->stats_cap = cap;
+    return MTDAO_OK;
+}
+
 static int enqueue_sync(mtdao_ctx *h, uint32_t mask) {
     SyncArgs a;
     std::memset(&a, 0, sizeof a);
@@ -497,6 +522,7 @@ extern "C" int mtdao_step(mtdao_handle h, const void *grads_dev, int32_t grad_dt
         e = launch_step(c->base, c->n_mom, grad_dtype, clip, a, h->num_sms, h->stream);
     }
     if (e != cudaSuccess) return cuda_fail(h, e, "step launch");
+    if (int rc = refresh_anchor(h, sync_mask)) return rc;
     ++h->step;
     return MTDAO_OK;
 }
@@ -555,9 +581,11 @@ extern "C" int mtdao_sync(mtdao_handle h, uint32_t mask) {
     if (int rc = check_handle(h)) return rc;
     if (mask >> h->n_states) return set_error(h, MTDAO_ERR_INVALID, "sync mask 0x%x has bits beyond "
                                               "the %d states", mask, h->n_states);
-    if (mask == 0 || h->M == 1) return MTDAO_OK;
+    if (mask == 0) return MTDAO_OK;
     if (int rc = select_device(h)) return rc;
-    return enqueue_sync(h, mask);
+    if (h->M > 1)
+        if (int rc = enqueue_sync(h, mask)) return rc;
+    return refresh_anchor(h, mask);
 }
 
 extern "C" int mtdao_sync_stats(mtdao_handle h, uint32_t mask, double *stats_dev) {
@@ -568,16 +596,7 @@ extern "C" int mtdao_sync_stats(mtdao_handle h, uint32_t mask, double *stats_dev
     if (h->M > 8) return set_error(h, MTDAO_ERR_INVALID, "diagnostics support M <= 8 (M = %d)", h->M);
     if (mask == 0) return MTDAO_OK;
     if (int rc = select_device(h)) return rc;
-    if (h->stats_partial == nullptr) {
-        const size_t cap = sync_stats_partial_capacity(h->num_sms, h->n_states, h->M);
-        cudaError_t e = cudaMalloc(reinterpret_cast<void **>(&h->stats_partial), cap * sizeof(double));
-        if (e != cudaSuccess) {
-            cudaGetLastError();
-            h->stats_partial = nullptr;
-            return set_error(h, MTDAO_ERR_OOM, "diagnostics workspace: %s", cudaGetErrorString(e));
-        }
-        h->stats_cap = cap;
-    }
+    if (int rc = ensure_stats_workspace(h)) return rc;
     SyncArgs a;
     std::memset(&a, 0, sizeof a);
     a.arena = h->arena;
@@ -588,6 +607,44 @@ extern "C" int mtdao_sync_stats(mtdao_handle h, uint32_t mask, double *stats_dev
         if (mask & (1u << s)) a.sel[a.n_sel++] = s;
     cudaError_t e = launch_sync_stats(a, h->num_sms, h->stats_partial, h->stats_cap, stats_dev, h->stream);
     if (e != cudaSuccess) return cuda_fail(h, e, "sync with diagnostics launch");
+    return refresh_anchor(h, mask);
+}
+
+extern "C" int mtdao_track_anchor(mtdao_handle h, int32_t enable) {
+    if (int rc = check_handle(h)) return rc;
+    if (int rc = select_device(h)) return rc;
+    if (!enable) {
+        if (h->anchor) {
+            cudaStreamSynchronize(h->stream);
+            cudaFree(h->anchor);
+            h->anchor = nullptr;
+        }
+        return MTDAO_OK;
+    }
+    if (h->anchor == nullptr) {
+        cudaError_t e = cudaMalloc(reinterpret_cast<void **>(&h->anchor),
+                                   static_cast<size_t>(h->n_padded) * sizeof(float));
+        if (e != cudaSuccess) {
+            cudaGetLastError();
+            h->anchor = nullptr;
+            return set_error(h, MTDAO_ERR_OOM, "anchor (%lld floats): %s",
+                             static_cast<long long>(h->n_padded), cudaGetErrorString(e));
+        }
+    }
+    return refresh_anchor(h, 1u);
+}
+
+extern "C" int mtdao_pseudo_grad_stats(mtdao_handle h, double *out_dev) {
+    if (int rc = check_handle(h)) return rc;
+    if (out_dev == nullptr) return set_error(h, MTDAO_ERR_INVALID, "out is NULL");
+    if (h->anchor == nullptr)
+        return set_error(h, MTDAO_ERR_STATE, "no anchor: call mtdao_track_anchor(h, 1) first");
+    if (h->M > 8) return set_error(h, MTDAO_ERR_INVALID, "diagnostics support M <= 8 (M = %d)", h->M);
+    if (int rc = select_device(h)) return rc;
+    if (int rc = ensure_stats_workspace(h)) return rc;
+    cudaError_t e = launch_pseudo_grad_stats(h->arena, h->anchor, h->n_padded, h->M, h->num_sms,
+                                             h->stats_partial, h->stats_cap, out_dev, h->stream);
+    if (e != cudaSuccess) return cuda_fail(h, e, "pseudo-gradient diagnostics launch");
     return MTDAO_OK;
 }
 

@@ -81,6 +81,13 @@ cudaError_t launch_grad_sqnorm(const void *grads, int grad_dtype, int32_t M, int
                                int blocks_per_replica, double *partial, double *out,
                                float *clip_scale, double rho, cudaStream_t stream);
 
+// Pseudo-gradient diagnostics of x[M][n] against anchor[n] into stats[2M+2]
+// (as documented for mtdao_pseudo_grad_stats); M must be 1..8.  Uses the
+// sync-diagnostics workspace.
+cudaError_t launch_pseudo_grad_stats(const float *x, const float *anchor, int64_t n, int M, int num_sms,
+                                     double *partial, size_t partial_cap, double *stats,
+                                     cudaStream_t stream);
+
 // Record a message for mtdao_last_error(NULL) in the calling thread and
 // return code (for entry points that have no handle).
 int set_thread_error(int code, const char *msg);

@@ -211,14 +211,15 @@ __global__ void __launch_bounds__(kThreads) sync_stats_kernel(const SyncArgs a, 
 }
 
 // stats[sel * Q + q] = sum over blocks of partial (in block order); q = 0 is
-// divided by M (the variance is a mean over workers).
-__global__ void sync_stats_finalize_kernel(const double *partial, int blocks, int Q, int M,
+// divided by divide_first (M for the variance, a mean over workers)
+// (divide_first = 0 leaves q = 0 undivided)
+__global__ void sync_stats_finalize_kernel(const double *partial, int blocks, int Q, int divide_first,
                                            double *stats) {
     const int sel = blockIdx.x, q = threadIdx.x;
     if (q >= Q) return;
     double total = 0.0;
     for (int b = 0; b < blocks; ++b) total += partial[(static_cast<int64_t>(sel) * blocks + b) * Q + q];
-    stats[sel * Q + q] = q == 0 ? total / M : total;
+    stats[sel * Q + q] = (q == 0 && divide_first > 0) ? total / divide_first : total;
 }
 
 template <int M>
@@ -240,7 +241,98 @@ cudaError_t launch_sync_stats_t(const SyncArgs &a, int num_sms, double *partial,
     return cudaGetLastError();
 }
 
+// Pseudo-gradient diagnostics of the parameters x[M][n] against the anchor
+// a[n] (the parameters at the last average), read-only, with fixed-order
+// sums into partial[block * Q + q], Q = 2M + 2:
+//   q = m          (x_m - a)^2
+//   q = M + m      (x_m - a) * (x_bar - a)
+//   q = 2M         (x_bar - a)^2
+//   q = 2M + 1     a^2
+// x_bar is the replica mean of replica_mean.cuh (the value an average would
+// store now).
+template <int M>
+__global__ void __launch_bounds__(kThreads) pseudo_grad_stats_kernel(const float *x, const float *anchor,
+                                                                     int64_t n, double *partial) {
+    constexpr int Q = 2 * M + 2;
+    const int64_t nv = n / 4;
+    Kahan acc[Q];
+    for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < nv;
+         i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+        const int64_t e = 4 * i;
+        float r[M][4], av[4];
+#pragma unroll
+        for (int m = 0; m < M; ++m) to_array(ld_state(x + m * n + e), r[m]);
+        to_array(__ldcs(reinterpret_cast<const float4 *>(anchor + e)), av);
+        float q[Q];
+#pragma unroll
+        for (int j = 0; j < Q; ++j) q[j] = 0.0f;
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+            const float mean = replica_mean<M>([&](int m) { return r[m][k]; });
+            const float glob = mean - av[k];
+            q[2 * M] = fmaf(glob, glob, q[2 * M]);
+            q[2 * M + 1] = fmaf(av[k], av[k], q[2 * M + 1]);
+#pragma unroll
+            for (int m = 0; m < M; ++m) {
+                const float loc = r[m][k] - av[k];
+                q[m] = fmaf(loc, loc, q[m]);
+                q[M + m] = fmaf(loc, glob, q[M + m]);
+            }
+        }
+#pragma unroll
+        for (int j = 0; j < Q; ++j) acc[j].add(q[j]);
+    }
+    __shared__ double part[Q][kThreads / 32];
+    const int w = threadIdx.x >> 5, l = threadIdx.x & 31;
+#pragma unroll
+    for (int j = 0; j < Q; ++j) {
+        const double v = warp_sum(acc[j].value());
+        if (l == 0) part[j][w] = v;
+    }
+    __syncthreads();
+    if (threadIdx.x < Q) {
+        double total = 0.0;
+        for (int i = 0; i < static_cast<int>(blockDim.x >> 5); ++i) total += part[threadIdx.x][i];
+        partial[static_cast<int64_t>(blockIdx.x) * Q + threadIdx.x] = total;
+    }
+}
+
+template <int M>
+cudaError_t launch_pseudo_grad_stats_t(const float *x, const float *anchor, int64_t n, int num_sms,
+                                       double *partial, size_t partial_cap, double *stats,
+                                       cudaStream_t stream) {
+    constexpr int Q = 2 * M + 2;
+    static const int per_sm = blocks_per_sm(pseudo_grad_stats_kernel<M>);
+    int64_t gx = static_cast<int64_t>(per_sm) * num_sms;
+    const int64_t need = (n / 4 + kThreads - 1) / kThreads;
+    if (gx > need) gx = need;
+    if (gx < 1) gx = 1;
+    if (static_cast<size_t>(gx) * Q > partial_cap) return cudaErrorInvalidValue;
+    pseudo_grad_stats_kernel<M><<<static_cast<unsigned>(gx), kThreads, 0, stream>>>(x, anchor, n, partial);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    // same fixed-order finalisation as the sync diagnostics, with no division
+    sync_stats_finalize_kernel<<<1, 32, 0, stream>>>(partial, static_cast<int>(gx), Q, 0, stats);
+    return cudaGetLastError();
+}
+
 }  // namespace
+
+cudaError_t launch_pseudo_grad_stats(const float *x, const float *anchor, int64_t n, int M, int num_sms,
+                                     double *partial, size_t partial_cap, double *stats,
+                                     cudaStream_t stream) {
+    switch (M) {
+        case 1: return launch_pseudo_grad_stats_t<1>(x, anchor, n, num_sms, partial, partial_cap, stats, stream);
+        case 2: return launch_pseudo_grad_stats_t<2>(x, anchor, n, num_sms, partial, partial_cap, stats, stream);
+        case 3: return launch_pseudo_grad_stats_t<3>(x, anchor, n, num_sms, partial, partial_cap, stats, stream);
+        case 4: return launch_pseudo_grad_stats_t<4>(x, anchor, n, num_sms, partial, partial_cap, stats, stream);
+        case 5: return launch_pseudo_grad_stats_t<5>(x, anchor, n, num_sms, partial, partial_cap, stats, stream);
+        case 6: return launch_pseudo_grad_stats_t<6>(x, anchor, n, num_sms, partial, partial_cap, stats, stream);
+        case 7: return launch_pseudo_grad_stats_t<7>(x, anchor, n, num_sms, partial, partial_cap, stats, stream);
+        case 8: return launch_pseudo_grad_stats_t<8>(x, anchor, n, num_sms, partial, partial_cap, stats, stream);
+        default: return cudaErrorNotSupported;
+    }
+}
 
 size_t sync_stats_partial_capacity(int num_sms, int n_states, int M) {
     // at most 16 resident blocks per SM of 256 threads, split over the states

@@ -105,3 +105,49 @@ def test_sync_stats_rejects_large_M_and_bad_masks(P):
     with pytest.raises(P.MTDAOError):
         P.mtdao_sync_stats(eng.h, 1 << 7, out.data_ptr())
     eng.close()
+
+
+@pytest.mark.parametrize("M", [2, 4, 8])
+def test_pseudo_grad_stats_against_oracle(P, M):
+    """Anchor = parameters at the last average; mid-round diagnostics of the
+    pseudo-gradients match the oracle's definitions on the same values."""
+    from oracle.oracle import pseudo_grad_stats
+    w = workload_dict([40000, 123], M, betas=(0.9, 0.999), px=8, pu=4, pv=8)
+    eng = P.MTDAO(w["opt"], M, w["shapes"])
+    eng.set_params(torch.randn(eng.n_padded, device="cuda") * 0.02)
+    eng.track_anchor(True)
+    gen = torch.Generator(device="cuda").manual_seed(M)
+    common = torch.randn(eng.n_padded, device="cuda", generator=gen)
+
+    def step():
+        g = common[None, :] + torch.randn((M, eng.n_padded), device="cuda", generator=gen)
+        eng.step(g.contiguous(), 1e-3)
+
+    for _ in range(8):
+        step()                                        # x averaged at the end of step 8
+    at_sync = eng.pseudo_grad_stats().cpu().numpy()
+    assert np.all(at_sync[:M] == 0) and at_sync[2 * M] == 0 and at_sync[2 * M + 1] > 0
+    anchor = eng.state_view(0)[0].cpu().numpy().astype(np.float64)
+    for _ in range(5):
+        step()
+    got = eng.pseudo_grad_stats().cpu().numpy()
+    x = eng.state_view(0).cpu().numpy().astype(np.float64)
+    ref = pseudo_grad_stats(x, anchor)
+    np.testing.assert_allclose(got, ref, rtol=1e-5)
+    cos = got[M:2 * M] / np.sqrt(got[:M] * got[2 * M])
+    assert np.all(cos > 0.3) and np.all(cos <= 1.0 + 1e-6)
+    eng.close()
+
+
+def test_pseudo_grad_stats_needs_an_anchor(P):
+    w = workload_dict([1024], 2, betas=(0.9,))
+    eng = P.MTDAO(w["opt"], 2, w["shapes"])
+    out = torch.zeros(8, dtype=torch.float64, device="cuda")
+    with pytest.raises(P.MTDAOError) as e:
+        P.mtdao_pseudo_grad_stats(eng.h, out.data_ptr())
+    assert e.value.code == P.ERR_STATE
+    eng.track_anchor(True)
+    eng.track_anchor(False)
+    with pytest.raises(P.MTDAOError):
+        P.mtdao_pseudo_grad_stats(eng.h, out.data_ptr())
+    eng.close()

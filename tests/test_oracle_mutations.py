@@ -55,6 +55,8 @@ MUTATIONS = {
     "variance_over_M_minus_1": ("out[0] += (v - mean) * (v - mean) / (double)M;",
                                 "out[0] += (v - mean) * (v - mean) / (double)(M - 1);"),
     "dot_with_worker_instead_of_mean": ("out[2 + M + m] += v * mean;", "out[2 + M + m] += v * v;"),
+    "global_pseudo_grad_without_anchor": ("double global = sum / (double)M - a[i];",
+                                          "double global = sum / (double)M;"),
 }
 
 

@@ -495,3 +495,23 @@ def test_state_stats_against_numpy_and_closed_forms():
     same = state_stats(np.tile(s[0], (3, 1)))
     assert 0.0 <= same[0] <= 1e-28 * same[1]
     np.testing.assert_allclose(same[1:], np.dot(s[0], s[0]), rtol=1e-14)
+
+
+def test_pseudo_grad_stats_against_numpy():
+    """Section 4.1 / 5.4: pseudo-gradients Delta^m = x^m - a over a round,
+    their mean, cosine similarity and the relative change of the model."""
+    from oracle.oracle import pseudo_grad_stats
+    rng = np.random.default_rng(18)
+    M, n = 4, 257
+    a = rng.standard_normal(n)
+    x = a[None, :] + 0.1 * rng.standard_normal((M, n)) + 0.05
+    out = pseudo_grad_stats(x, a)
+    loc = x - a[None, :]
+    glob = x.mean(axis=0) - a
+    np.testing.assert_allclose(out[:M], np.sum(loc * loc, axis=1), rtol=1e-13)
+    np.testing.assert_allclose(out[M:2 * M], loc @ glob, rtol=1e-12)
+    assert abs(out[2 * M] - glob @ glob) < 1e-12 * out[2 * M]
+    assert abs(out[2 * M + 1] - a @ a) < 1e-13 * out[2 * M + 1]
+    # all workers moved identically: every cosine is 1, mean move = each move
+    same = pseudo_grad_stats(np.tile(x[0], (3, 1)), a)
+    np.testing.assert_allclose(same[3:6] / np.sqrt(same[:3] * same[6]), 1.0, rtol=1e-12)
