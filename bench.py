@@ -59,6 +59,29 @@ def parse_args():
     return ap.parse_args()
 
 
+def rank_env():
+    """(rank, world size, local rank) from the torchrun environment."""
+    return (int(os.environ.get("RANK", "0")), int(os.environ.get("WORLD_SIZE", "1")),
+            int(os.environ.get("LOCAL_RANK", "0")))
+
+
+def max_over_ranks(value: float, dist=None, device="cpu") -> float:
+    """The largest value over all ranks (a job takes as long as its slowest
+    rank); the identity without a process group."""
+    if dist is None:
+        return value
+    import torch
+    t = torch.tensor([value], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_rate(units_per_rank: float, world: int, seconds: float) -> float:
+    """Whole-job throughput: every rank processes its own units (weak
+    scaling, no data-path collective), in the slowest rank's time."""
+    return world * units_per_rank / seconds
+
+
 def round_len(opt) -> int:
     periods = [opt["period_x"], opt.get("period_v", 0)] + list(opt["period_u"])
     return max(p for p in periods if p > 0)
@@ -199,7 +222,7 @@ def oracle_sample_rate(w, n_sample: int, rounds: int = 1):
 
 
 def run_reference(args):
-    rank = int(os.environ.get("RANK", "0"))
+    rank, _, _ = rank_env()
     if rank != 0:
         return 0
     w = W.get(args.workload)
@@ -245,9 +268,7 @@ def run_ours(args):
     import paper_2510_05361_gb300 as P
     from synth.device import DeviceInputs
 
-    rank = int(os.environ.get("RANK", "0"))
-    world = int(os.environ.get("WORLD_SIZE", "1"))
-    local = int(os.environ.get("LOCAL_RANK", "0"))
+    rank, world, local = rank_env()
     torch.cuda.set_device(local)
     dist = None
     if world > 1:
@@ -318,13 +339,8 @@ def run_ours(args):
     if small:
         # L2 was flushed before every launch; time only the launches.
         elapsed_ms = sum(ms for rnd in launch_ms for ms in rnd)
-    if dist is not None:
-        t = torch.tensor([elapsed_ms], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        elapsed_ms = float(t.item())
-
-    units = world * M * n * H * args.steps
-    value = units / (elapsed_ms / 1e3)
+    elapsed_ms = max_over_ranks(elapsed_ms, dist, "cuda")
+    value = job_rate(M * n * H * args.steps, world, elapsed_ms / 1e3)
     step_ms = statistics.mean(plain)
     peak, peak_kind = hbm_peak()
     achieved = step_bytes / (step_ms / 1e3) / 1e9
@@ -394,12 +410,8 @@ def run_ours(args):
                 P.mtdao_step_host(eng.h, host_g.data_ptr(), gdt, opt["lr"], eng.sync_due())
             P.mtdao_copy_state_to_host(eng.h, 0, 0, host_x.data_ptr())   # round's synced x
         torch.cuda.synchronize()
-        e2e_s = time.perf_counter() - t0
-        if dist is not None:
-            t = torch.tensor([e2e_s], device="cuda")
-            dist.all_reduce(t, op=dist.ReduceOp.MAX)
-            e2e_s = float(t.item())
-        e2e = {"value": world * M * n * H * args.e2e_rounds / e2e_s, "unit": "params/s",
+        e2e_s = max_over_ranks(time.perf_counter() - t0, dist, "cuda")
+        e2e = {"value": job_rate(M * n * H * args.e2e_rounds, world, e2e_s), "unit": "params/s",
                "h2d_bytes_per_step": H * M * n * g_bytes, "d2h_bytes_per_step": n * 4,
                "rounds": args.e2e_rounds}
         del host_g

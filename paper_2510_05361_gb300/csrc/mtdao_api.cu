@@ -223,8 +223,9 @@ StepScalars step_scalars(const mtdao_config *c, int64_t t, double lr) {
 }
 
 // Allocation with optional fault injection: MTDAO_FAULT_ALLOC=k makes the
-// k-th device allocation of a create (1-based) report out-of-memory.
-int g_alloc_counter = 0;
+// k-th device allocation of a create (1-based) report out-of-memory.  The
+// counter is per thread, so concurrent creates do not disturb each other.
+thread_local int g_alloc_counter = 0;
 
 cudaError_t dev_alloc(void **p, size_t bytes) {
     ++g_alloc_counter;
