@@ -224,10 +224,13 @@ int mtdao_step_host(mtdao_handle h, const void *grads_host, int32_t grad_dtype, 
 /*
  * Outer synchronisation (Algorithms 1-3, E_m[.] with OuterOpt = averaging):
  * every state in mask is replaced, on every replica, by the equal-weight
- * mean over the M replicas.  Computed in fp32 as s_0 + S / M with S the
- * Kahan-compensated sum of (s_m - s_0) in replica order, which returns s_0
- * bit for bit when the replicas agree; the fused average in mtdao_step and
- * mtdao_sync_stats use the same routine.  mask 0 is a no-op.
+ * mean over the M replicas.  Computed in fp32 as s_0 + (A + B) / M, A and
+ * B the Kahan-compensated sums of (s_m - s_0) over replicas 1..h-1 and
+ * h..M-1 (h = floor(M/2)), each in replica order; this returns s_0 bit for
+ * bit when the replicas agree and stays within about one rounding of the
+ * exact mean for any M.  The fused average in mtdao_step and
+ * mtdao_sync_stats use the same routine (identical bits).  mask 0 is a
+ * no-op.
  */
 int mtdao_sync(mtdao_handle h, uint32_t mask);
 
