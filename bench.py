@@ -379,19 +379,19 @@ def run_ours(args):
     # pseudo-gradient diagnostics: a read-only pass over x and the anchor
     pg_ms = []
     if M <= 8:
-        P.mtdao_track_anchor(eng.h, True)
+        P.mtdao_track_anchor(eng.h, 1)
         pg_out = torch.empty((2 * M + 2,), dtype=torch.float64, device="cuda")
         for i in range(6):
             a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
             if flush is not None:
                 flush.fill_(1.0)
             a.record(stream)
-            P.mtdao_pseudo_grad_stats(eng.h, pg_out.data_ptr())
+            P.mtdao_pseudo_grad_stats(eng.h, 0, pg_out.data_ptr())
             b.record(stream)
             torch.cuda.synchronize()
             if i >= 2:
                 pg_ms.append(a.elapsed_time(b))
-        P.mtdao_track_anchor(eng.h, False)
+        P.mtdao_track_anchor(eng.h, 0)
     pg_bytes = (M + 1) * n * 4
 
     # end to end through the host-buffer C-ABI call

@@ -253,31 +253,33 @@ int mtdao_sync(mtdao_handle h, uint32_t mask);
 int mtdao_sync_stats(mtdao_handle h, uint32_t mask, double *stats_dev);
 
 /*
- * Anchor tracking for pseudo-gradient diagnostics (section 4.1 "Other
- * Metrics"; section 5.4's worker update over a round, the pseudo-gradient
- * Delta^m = x^m_{t+K} - x^m_t).  enable != 0 allocates one [n_padded] fp32
- * vector and sets it to replica 0's x; from then on every step, sync or
- * sync_stats whose mask includes x (bit 0) copies replica 0's x into it
- * after the average, so it holds the parameters at the start of the current
- * round (one device-to-device copy of n_padded floats per parameter
- * average).  enable == 0 frees it (synchronises the stream).
+ * Anchors for the diagnostics of change over a round (section 4.1 "Other
+ * Metrics": relative change ||s_{t+K} - s_t|| / ||s_t||; section 5.4: the
+ * pseudo-gradient Delta^m = x^m_{t+K} - x^m_t, the worker update over a
+ * round, and its mean).  Bit s of state_mask keeps an anchor for state s:
+ * one [n_padded] fp32 vector, set to replica 0's value now and, from then
+ * on, after every step, sync or sync_stats that averages state s (one
+ * device-to-device copy of n_padded floats per average), so it holds the
+ * state at the start of the current round.  Anchors whose bit is clear are
+ * freed (synchronises the stream); state_mask 0 frees all.
  */
-int mtdao_track_anchor(mtdao_handle h, int32_t enable);
+int mtdao_track_anchor(mtdao_handle h, uint32_t state_mask);
 
 /*
- * Pseudo-gradient diagnostics of the current parameters against the anchor
- * a, read-only (no state changes), fixed-order sums.  With x_bar the replica
- * mean an average would store now, out_dev (device, 2M + 2 doubles) gets
- *   [m]        ||x_m - a||^2                 m = 0..M-1  (local pseudo-gradient)
- *   [M + m]    <x_m - a, x_bar - a>
- *   [2M]       ||x_bar - a||^2                           (global pseudo-gradient)
+ * Change diagnostics of one state against its anchor a, read-only (no state
+ * changes), fixed-order sums.  With s_bar the replica mean an average would
+ * store now, out_dev (device, 2M + 2 doubles) gets
+ *   [m]        ||s_m - a||^2                 m = 0..M-1  (local change, for x
+ *                                                          the pseudo-gradient)
+ *   [M + m]    <s_m - a, s_bar - a>
+ *   [2M]       ||s_bar - a||^2                           (global change)
  *   [2M + 1]   ||a||^2
  * so cos(local, global) = [M+m] / sqrt([m] [2M]) and the relative change of
- * the averaged model over the round = sqrt([2M] / [2M+1]).  Call it before
- * the round's parameter average.  MTDAO_ERR_STATE without an anchor;
- * requires M <= 8.
+ * the averaged state over the round = sqrt([2M] / [2M+1]).  Call it before
+ * the round's average of that state.  MTDAO_ERR_STATE if the state has no
+ * anchor; requires M <= 8.
  */
-int mtdao_pseudo_grad_stats(mtdao_handle h, double *out_dev);
+int mtdao_pseudo_grad_stats(mtdao_handle h, int32_t state, double *out_dev);
 
 /* Mask of states due at the end of the next step (mtdao_due_mask at t). */
 int mtdao_sync_due(mtdao_handle h, uint32_t *mask_out);

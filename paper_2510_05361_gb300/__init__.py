@@ -84,8 +84,8 @@ def _load():
         "mtdao_sync": (ctypes.c_int, [H, ctypes.c_uint32]),
         "mtdao_sync_due": (ctypes.c_int, [H, ctypes.POINTER(ctypes.c_uint32)]),
         "mtdao_sync_stats": (ctypes.c_int, [H, ctypes.c_uint32, ctypes.c_void_p]),
-        "mtdao_track_anchor": (ctypes.c_int, [H, ctypes.c_int32]),
-        "mtdao_pseudo_grad_stats": (ctypes.c_int, [H, ctypes.c_void_p]),
+        "mtdao_track_anchor": (ctypes.c_int, [H, ctypes.c_uint32]),
+        "mtdao_pseudo_grad_stats": (ctypes.c_int, [H, ctypes.c_int32, ctypes.c_void_p]),
         "mtdao_grad_sqnorm": (ctypes.c_int, [H, ctypes.c_void_p, ctypes.c_int32, ctypes.c_void_p]),
         "mtdao_grad_sqnorm_static": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_int32, ctypes.c_int32,
                                                     ctypes.c_int64, ctypes.c_void_p, ctypes.c_void_p]),
@@ -227,12 +227,12 @@ def mtdao_sync_stats(h, mask: int, stats_dev_ptr: int) -> None:
     _check(lib.mtdao_sync_stats(h, mask, ctypes.c_void_p(stats_dev_ptr)), h)
 
 
-def mtdao_track_anchor(h, enable: bool) -> None:
-    _check(lib.mtdao_track_anchor(h, 1 if enable else 0), h)
+def mtdao_track_anchor(h, state_mask: int) -> None:
+    _check(lib.mtdao_track_anchor(h, int(state_mask)), h)
 
 
-def mtdao_pseudo_grad_stats(h, out_dev_ptr: int) -> None:
-    _check(lib.mtdao_pseudo_grad_stats(h, ctypes.c_void_p(out_dev_ptr)), h)
+def mtdao_pseudo_grad_stats(h, state: int, out_dev_ptr: int) -> None:
+    _check(lib.mtdao_pseudo_grad_stats(h, int(state), ctypes.c_void_p(out_dev_ptr)), h)
 
 
 def mtdao_sync_due(h) -> int:
@@ -363,15 +363,17 @@ class MTDAO:
         mtdao_sync_stats(self.h, mask, out.data_ptr())
         return out
 
-    def track_anchor(self, enable: bool = True) -> None:
-        mtdao_track_anchor(self.h, enable)
+    def track_anchor(self, state_mask: int = 1) -> None:
+        """Keep anchors for the states in state_mask (bit 0 = x); 0 frees all."""
+        mtdao_track_anchor(self.h, state_mask)
 
-    def pseudo_grad_stats(self):
-        """Pseudo-gradient diagnostics against the anchor as a device tensor
-        [2M + 2] (see mtdao_pseudo_grad_stats)."""
+    def pseudo_grad_stats(self, state: int = 0):
+        """Change diagnostics of one state against its anchor as a device
+        tensor [2M + 2] (see mtdao_pseudo_grad_stats); state 0 gives the
+        pseudo-gradients."""
         import torch
         out = torch.empty((2 * self.M + 2,), dtype=torch.float64, device="cuda")
-        mtdao_pseudo_grad_stats(self.h, out.data_ptr())
+        mtdao_pseudo_grad_stats(self.h, state, out.data_ptr())
         return out
 
     def state_ptr(self, state: int, replica: int) -> int:

@@ -78,7 +78,7 @@ struct mtdao_ctx {
     int norm_blocks = 1;
     double *stats_partial = nullptr;  // diagnostics workspace (allocated on first use)
     size_t stats_cap = 0;
-    float *anchor = nullptr;          // x at the last parameter average (mtdao_track_anchor)
+    float *anchor[2 + MTDAO_MAX_MOM] = {};  // per state: its value at the last average
     // host-gradient staging (mtdao_step_host)
     void *staging[2] = {nullptr, nullptr};
     size_t staging_bytes = 0;
@@ -253,7 +253,8 @@ void release(mtdao_ctx *h) {
     if (h->norm_out) cudaFree(h->norm_out);
     if (h->norm_partial) cudaFree(h->norm_partial);
     if (h->stats_partial) cudaFree(h->stats_partial);
-    if (h->anchor) cudaFree(h->anchor);
+    for (float *a : h->anchor)
+        if (a) cudaFree(a);
 }
 
 int check_handle(mtdao_ctx *h) {
@@ -441,13 +442,16 @@ extern "C" int mtdao_set_params(mtdao_handle h, const float *x0_dev) {
 
 // ====================================================================== hot path
 
-// After a step or sync whose mask includes x (bit 0), the tracked anchor
-// becomes the averaged parameters (replica 0's copy).
+// After a step or sync that averaged the states in mask, each tracked
+// anchor among them becomes the averaged value (replica 0's copy).
 static int refresh_anchor(mtdao_ctx *h, uint32_t mask) {
-    if (h->anchor == nullptr || (mask & 1u) == 0) return MTDAO_OK;
-    cudaError_t e = cudaMemcpyAsync(h->anchor, h->arena, static_cast<size_t>(h->n_padded) * sizeof(float),
-                                    cudaMemcpyDeviceToDevice, h->stream);
-    if (e != cudaSuccess) return cuda_fail(h, e, "anchor copy");
+    for (int s = 0; s < h->n_states; ++s) {
+        if (h->anchor[s] == nullptr || ((mask >> s) & 1u) == 0) continue;
+        const float *src = h->arena + static_cast<int64_t>(s) * h->M * h->n_padded;
+        cudaError_t e = cudaMemcpyAsync(h->anchor[s], src, static_cast<size_t>(h->n_padded) * sizeof(float),
+                                        cudaMemcpyDeviceToDevice, h->stream);
+        if (e != cudaSuccess) return cuda_fail(h, e, "anchor copy");
+    }
     return MTDAO_OK;
 }
 
@@ -611,41 +615,50 @@ extern "C" int mtdao_sync_stats(mtdao_handle h, uint32_t mask, double *stats_dev
     return refresh_anchor(h, mask);
 }
 
-extern "C" int mtdao_track_anchor(mtdao_handle h, int32_t enable) {
+extern "C" int mtdao_track_anchor(mtdao_handle h, uint32_t state_mask) {
     if (int rc = check_handle(h)) return rc;
+    if (state_mask >> h->n_states)
+        return set_error(h, MTDAO_ERR_INVALID, "state mask 0x%x has bits beyond the %d states", state_mask,
+                         h->n_states);
     if (int rc = select_device(h)) return rc;
-    if (!enable) {
-        if (h->anchor) {
-            cudaStreamSynchronize(h->stream);
-            cudaFree(h->anchor);
-            h->anchor = nullptr;
+    bool synced = false;
+    for (int s = 0; s < h->n_states; ++s) {
+        const bool want = (state_mask >> s) & 1u;
+        if (!want && h->anchor[s] != nullptr) {
+            if (!synced) {
+                cudaStreamSynchronize(h->stream);
+                synced = true;
+            }
+            cudaFree(h->anchor[s]);
+            h->anchor[s] = nullptr;
+        } else if (want && h->anchor[s] == nullptr) {
+            cudaError_t e = cudaMalloc(reinterpret_cast<void **>(&h->anchor[s]),
+                                       static_cast<size_t>(h->n_padded) * sizeof(float));
+            if (e != cudaSuccess) {
+                cudaGetLastError();
+                h->anchor[s] = nullptr;
+                return set_error(h, MTDAO_ERR_OOM, "anchor of state %d (%lld floats): %s", s,
+                                 static_cast<long long>(h->n_padded), cudaGetErrorString(e));
+            }
+            if (int rc = refresh_anchor(h, 1u << s)) return rc;
         }
-        return MTDAO_OK;
     }
-    if (h->anchor == nullptr) {
-        cudaError_t e = cudaMalloc(reinterpret_cast<void **>(&h->anchor),
-                                   static_cast<size_t>(h->n_padded) * sizeof(float));
-        if (e != cudaSuccess) {
-            cudaGetLastError();
-            h->anchor = nullptr;
-            return set_error(h, MTDAO_ERR_OOM, "anchor (%lld floats): %s",
-                             static_cast<long long>(h->n_padded), cudaGetErrorString(e));
-        }
-    }
-    return refresh_anchor(h, 1u);
+    return MTDAO_OK;
 }
 
-extern "C" int mtdao_pseudo_grad_stats(mtdao_handle h, double *out_dev) {
+extern "C" int mtdao_pseudo_grad_stats(mtdao_handle h, int32_t state, double *out_dev) {
     if (int rc = check_handle(h)) return rc;
     if (out_dev == nullptr) return set_error(h, MTDAO_ERR_INVALID, "out is NULL");
-    if (h->anchor == nullptr)
-        return set_error(h, MTDAO_ERR_STATE, "no anchor: call mtdao_track_anchor(h, 1) first");
+    if (state < 0 || state >= h->n_states) return set_error(h, MTDAO_ERR_INVALID, "state %d out of range", state);
+    if (h->anchor[state] == nullptr)
+        return set_error(h, MTDAO_ERR_STATE, "state %d has no anchor: track it with mtdao_track_anchor", state);
     if (h->M > 8) return set_error(h, MTDAO_ERR_INVALID, "diagnostics support M <= 8 (M = %d)", h->M);
     if (int rc = select_device(h)) return rc;
     if (int rc = ensure_stats_workspace(h)) return rc;
-    cudaError_t e = launch_pseudo_grad_stats(h->arena, h->anchor, h->n_padded, h->M, h->num_sms,
+    const float *x = h->arena + static_cast<int64_t>(state) * h->M * h->n_padded;
+    cudaError_t e = launch_pseudo_grad_stats(x, h->anchor[state], h->n_padded, h->M, h->num_sms,
                                              h->stats_partial, h->stats_cap, out_dev, h->stream);
-    if (e != cudaSuccess) return cuda_fail(h, e, "pseudo-gradient diagnostics launch");
+    if (e != cudaSuccess) return cuda_fail(h, e, "change diagnostics launch");
     return MTDAO_OK;
 }
 

@@ -115,7 +115,7 @@ def test_pseudo_grad_stats_against_oracle(P, M):
     w = workload_dict([40000, 123], M, betas=(0.9, 0.999), px=8, pu=4, pv=8)
     eng = P.MTDAO(w["opt"], M, w["shapes"])
     eng.set_params(torch.randn(eng.n_padded, device="cuda") * 0.02)
-    eng.track_anchor(True)
+    eng.track_anchor(0b011)                           # x and u1
     gen = torch.Generator(device="cuda").manual_seed(M)
     common = torch.randn(eng.n_padded, device="cuda", generator=gen)
 
@@ -124,18 +124,22 @@ def test_pseudo_grad_stats_against_oracle(P, M):
         eng.step(g.contiguous(), 1e-3)
 
     for _ in range(8):
-        step()                                        # x averaged at the end of step 8
-    at_sync = eng.pseudo_grad_stats().cpu().numpy()
+        step()                                        # x and u1 averaged at the end of step 8
+    at_sync = eng.pseudo_grad_stats(0).cpu().numpy()
     assert np.all(at_sync[:M] == 0) and at_sync[2 * M] == 0 and at_sync[2 * M + 1] > 0
-    anchor = eng.state_view(0)[0].cpu().numpy().astype(np.float64)
-    for _ in range(5):
-        step()
-    got = eng.pseudo_grad_stats().cpu().numpy()
-    x = eng.state_view(0).cpu().numpy().astype(np.float64)
-    ref = pseudo_grad_stats(x, anchor)
-    np.testing.assert_allclose(got, ref, rtol=1e-5)
-    cos = got[M:2 * M] / np.sqrt(got[:M] * got[2 * M])
-    assert np.all(cos > 0.3) and np.all(cos <= 1.0 + 1e-6)
+    anchors = {s: eng.state_view(s)[0].cpu().numpy().astype(np.float64) for s in (0, 1)}
+    for _ in range(3):
+        step()                                        # steps 9-11: no average due
+    for s in (0, 1):
+        got = eng.pseudo_grad_stats(s).cpu().numpy()
+        cur = eng.state_view(s).cpu().numpy().astype(np.float64)
+        np.testing.assert_allclose(got, pseudo_grad_stats(cur, anchors[s]), rtol=1e-5)
+        cos = got[M:2 * M] / np.sqrt(got[:M] * got[2 * M])
+        assert np.all(cos > 0.3) and np.all(cos <= 1.0 + 1e-6)
+    step()                                            # step 12 averages u1: new u1 anchor
+    assert np.all(eng.pseudo_grad_stats(1).cpu().numpy()[:M] == 0)
+    with pytest.raises(P.MTDAOError):
+        eng.pseudo_grad_stats(2)                      # u2 has no anchor
     eng.close()
 
 
@@ -144,10 +148,13 @@ def test_pseudo_grad_stats_needs_an_anchor(P):
     eng = P.MTDAO(w["opt"], 2, w["shapes"])
     out = torch.zeros(8, dtype=torch.float64, device="cuda")
     with pytest.raises(P.MTDAOError) as e:
-        P.mtdao_pseudo_grad_stats(eng.h, out.data_ptr())
+        P.mtdao_pseudo_grad_stats(eng.h, 0, out.data_ptr())
     assert e.value.code == P.ERR_STATE
-    eng.track_anchor(True)
-    eng.track_anchor(False)
+    eng.track_anchor(0b1)
+    eng.track_anchor(0)
     with pytest.raises(P.MTDAOError):
-        P.mtdao_pseudo_grad_stats(eng.h, out.data_ptr())
+        P.mtdao_pseudo_grad_stats(eng.h, 0, out.data_ptr())
+    with pytest.raises(P.MTDAOError) as e:
+        P.mtdao_track_anchor(eng.h, 1 << 5)
+    assert e.value.code == P.ERR_INVALID
     eng.close()
