@@ -210,6 +210,19 @@ int mtdao_step(mtdao_handle h, const void *grads_dev, int32_t grad_dtype, double
                uint32_t sync_mask);
 
 /*
+ * count consecutive local steps in one call, each with the averages its end
+ * brings under the handle's schedule (mtdao_due_mask at the handle's t):
+ * the same work as count pairs of mtdao_sync_due + mtdao_step, without a
+ * round trip to the caller per step (for small models, whose steps take
+ * tens of microseconds).  Step k reads its gradients at
+ * grads_dev + k * grads_stride_bytes (stride 0: the same buffer for every
+ * step; otherwise a multiple of 16) and uses lrs[k] (host array of count
+ * doubles).  Stops at the first failing step (t counts the steps done).
+ */
+int mtdao_run(mtdao_handle h, const void *grads_dev, int64_t grads_stride_bytes, int32_t grad_dtype,
+              const double *lrs, int32_t count);
+
+/*
  * mtdao_step with the gradients in host memory ([M][n_padded], 16-byte
  * aligned).  Pinned memory (cudaHostAlloc / cudaHostRegister) is read by the
  * step kernel directly over the host link, with no copy and no staging

@@ -81,6 +81,8 @@ def _load():
                                       ctypes.c_uint32]),
         "mtdao_step_host": (ctypes.c_int, [H, ctypes.c_void_p, ctypes.c_int32, ctypes.c_double,
                                            ctypes.c_uint32]),
+        "mtdao_run": (ctypes.c_int, [H, ctypes.c_void_p, ctypes.c_int64, ctypes.c_int32,
+                                     ctypes.POINTER(ctypes.c_double), ctypes.c_int32]),
         "mtdao_sync": (ctypes.c_int, [H, ctypes.c_uint32]),
         "mtdao_sync_due": (ctypes.c_int, [H, ctypes.POINTER(ctypes.c_uint32)]),
         "mtdao_sync_stats": (ctypes.c_int, [H, ctypes.c_uint32, ctypes.c_void_p]),
@@ -215,6 +217,13 @@ def mtdao_step(h, grads_dev_ptr: int, grad_dtype: int, lr: float, sync_mask: int
     _check(lib.mtdao_step(h, ctypes.c_void_p(grads_dev_ptr), grad_dtype, float(lr), sync_mask), h)
 
 
+def mtdao_run(h, grads_dev_ptr: int, grads_stride_bytes: int, grad_dtype: int, lrs) -> None:
+    lrs = [float(v) for v in lrs]
+    arr = (ctypes.c_double * len(lrs))(*lrs)
+    _check(lib.mtdao_run(h, ctypes.c_void_p(grads_dev_ptr), int(grads_stride_bytes), grad_dtype, arr,
+                         len(lrs)), h)
+
+
 def mtdao_step_host(h, grads_host_ptr: int, grad_dtype: int, lr: float, sync_mask: int = 0) -> None:
     _check(lib.mtdao_step_host(h, ctypes.c_void_p(grads_host_ptr), grad_dtype, float(lr), sync_mask), h)
 
@@ -347,6 +356,16 @@ class MTDAO:
             dtype = BF16 if grads_host.dtype == torch.bfloat16 else F32
         mtdao_step_host(self.h, self._ptr(grads_host), dtype, lr, sync_mask)
         return sync_mask
+
+    def run(self, grads, lrs, dtype: int | None = None) -> None:
+        """len(lrs) local steps in one call.  grads: a [count][M][n_padded]
+        tensor (one buffer per step) or a [M][n_padded] tensor reused by
+        every step."""
+        if dtype is None:
+            import torch
+            dtype = BF16 if grads.dtype == torch.bfloat16 else F32
+        stride = grads.stride(0) * grads.element_size() if grads.dim() == 3 else 0
+        mtdao_run(self.h, self._ptr(grads), stride, dtype, lrs)
 
     def sync(self, mask: int) -> None:
         mtdao_sync(self.h, mask)

@@ -532,6 +532,20 @@ extern "C" int mtdao_step(mtdao_handle h, const void *grads_dev, int32_t grad_dt
     return MTDAO_OK;
 }
 
+extern "C" int mtdao_run(mtdao_handle h, const void *grads_dev, int64_t grads_stride_bytes,
+                         int32_t grad_dtype, const double *lrs, int32_t count) {
+    if (int rc = check_handle(h)) return rc;
+    if (count < 0 || (count > 0 && (grads_dev == nullptr || lrs == nullptr)))
+        return set_error(h, MTDAO_ERR_INVALID, "run: bad count or NULL arguments");
+    if (grads_stride_bytes < 0 || grads_stride_bytes % 16 != 0)
+        return set_error(h, MTDAO_ERR_ALIGN, "run: gradient stride must be a non-negative multiple of 16");
+    for (int32_t k = 0; k < count; ++k) {
+        const void *g = static_cast<const char *>(grads_dev) + static_cast<int64_t>(k) * grads_stride_bytes;
+        if (int rc = mtdao_step(h, g, grad_dtype, lrs[k], due_mask(&h->cfg, h->step))) return rc;
+    }
+    return MTDAO_OK;
+}
+
 extern "C" int mtdao_step_host(mtdao_handle h, const void *grads_host, int32_t grad_dtype, double lr,
                                uint32_t sync_mask) {
     if (int rc = check_handle(h)) return rc;

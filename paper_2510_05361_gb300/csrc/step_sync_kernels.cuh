@@ -1,11 +1,11 @@
 // step_sync_kernels.cuh -- the local step with the replica average fused in.
 //
-// step_sync_kernel is element-major: a lane updates the same 4 elements of
+// step_sync_kernel is element-major: a lane updates the same few elements of
 // all M replicas (M <= 4) or, for M = 8, of 4 replicas while the lane 16
-// places away holds the other 4, with the update of step_kernels.cuh; then
-// it writes each state due for averaging as the replica mean (E_m[.] of
-// Algorithms 1-3) instead of the local values.  The average costs no HBM
-// traffic beyond the step's own.
+// places away holds the other 4 (see FusedShape), with the update of
+// step_kernels.cuh; then it writes each state due for averaging as the
+// replica mean (E_m[.] of Algorithms 1-3) instead of the local values.  The
+// average costs no HBM traffic beyond the step's own.
 #pragma once
 
 #include "replica_mean.cuh"
@@ -26,7 +26,7 @@ namespace mtdao {
 //           4..7, and combine their parts of the average by shuffles.
 // Measured on the flat 2^27 sweep (GB/s of the fused step, Adam, f32):
 // issuing all loads first lifts M = 4 from ~6180 to ~6480 (the plain step's
-// level) but costs M = 2 (6650 -> 6500) and M = 8 (5840 -> 5000-5760,
+// level) but costs M = 2 (6650 -> 6500) and M = 8 (about 6050 -> 5000-5760,
 // register spills), hence the split.
 template <int M>
 struct FusedShape {

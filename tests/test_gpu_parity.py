@@ -380,3 +380,29 @@ def test_zero_learning_rate_leaves_parameters_bitwise(P):
     got = eng.state_view(0).cpu().numpy()
     assert np.array_equal(got.view(np.uint32), np.tile(x0, (4, 1)).view(np.uint32))
     eng.close()
+
+
+def test_run_equals_step_by_step(P):
+    """mtdao_run over a stack of gradient buffers (and with one reused
+    buffer) gives the bits of the same steps issued one by one."""
+    w = workload_dict(RAGGED, 4, betas=(0.9, 0.999), px=3, pu=2, pv=3)
+    lay = W.layout(w["shapes"])
+    idx = np.arange(lay["n_padded"])
+    x0 = torch.from_numpy(G.init_params(w, lay, SEED_I, idx)).cuda()
+    gs = torch.from_numpy(np.stack([host_grads(w, lay, SEED_G, t, idx) for t in range(7)])).cuda()
+    lrs = [1e-3 * (1 + 0.1 * t) for t in range(7)]
+    a, b, c, d = (P.MTDAO(w["opt"], 4, w["shapes"]) for _ in range(4))
+    for e in (a, b, c, d):
+        e.set_params(x0)
+    for t in range(7):
+        a.step(gs[t], lrs[t])
+        c.step(gs[0], lrs[t])
+    b.run(gs, lrs)
+    d.run(gs[0], lrs)
+    torch.cuda.synchronize()
+    assert b.t == 7 and d.t == 7
+    for s in range(a.n_states):
+        assert torch.equal(a.state_view(s), b.state_view(s)), s
+        assert torch.equal(c.state_view(s), d.state_view(s)), s
+    for e in (a, b, c, d):
+        e.close()
