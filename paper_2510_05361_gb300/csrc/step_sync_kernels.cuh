@@ -26,7 +26,7 @@ namespace mtdao {
 //           4..7, and combine their parts of the average by shuffles.
 // Measured on the flat 2^27 sweep (GB/s of the fused step, Adam, f32):
 // issuing all loads first lifts M = 4 from ~6180 to ~6480 (the plain step's
-// level) but costs M = 2 (6650 -> 6500) and M = 8 (about 6050 -> 5000-5760,
+// level) but costs M = 2 (6650 -> 6500) and M = 8 (about 6070 -> 5540-6030,
 // register spills), hence the split.
 template <int M>
 struct FusedShape {
