@@ -21,13 +21,17 @@ namespace mtdao {
 //           states are loaded, updated and stored one after another.
 //   M = 4 : one lane group, R = 4, V = 2 (64-bit accesses); every load of
 //           the chunk is issued before any arithmetic, as in step_kernel.
-//   M = 8 : two lane groups (half-warps), R = 4, V = 4, state by state;
-//           lanes q and q + 16 hold the same elements, replicas 0..3 and
-//           4..7, and combine their parts of the average by shuffles.
+//   M = 8 : two lane groups (half-warps), R = 4, V = 4, state by state with
+//           a lookahead: the next state's loads are issued before the
+//           current state is updated and stored, so two states' loads are
+//           in flight; lanes q and q + 16 hold the same elements, replicas
+//           0..3 and 4..7, and combine their parts of the average by
+//           shuffles.
 // Measured on the flat 2^27 sweep (GB/s of the fused step, Adam, f32):
 // issuing all loads first lifts M = 4 from ~6180 to ~6480 (the plain step's
-// level) but costs M = 2 (6650 -> 6500) and M = 8 (about 6070 -> 5540-6030,
-// register spills), hence the split.
+// level) but costs M = 2 (6650 -> 6500) and M = 8 (register spills); the
+// one-state lookahead lifts M = 8 from 6030-6065 to 6485-6727 (ADOPT with
+// bf16 gradients: 5439 -> 6089) and leaves M = 2 unchanged.
 template <int M>
 struct FusedShape {
     static constexpr int G = M == 8 ? 2 : 1;      // lane groups per warp
@@ -36,7 +40,19 @@ struct FusedShape {
     static constexpr int V = kPrefetch ? 2 : 4;   // elements per lane
     static constexpr int kLanes = 32 / G;         // lanes per group
     static constexpr int kChunk = kLanes * V;     // elements per warp iteration
+    static constexpr bool kLookahead = M == 8;    // state by state, next state's loads early
 };
+
+// Order in which the state-by-state shapes visit the states (arena index
+// 0 = x, 1 + j = u_j, 1 + N = v): ADOPT takes v first (it normalises the
+// gradient), Adam takes v after the momenta (it divides their combination),
+// x comes last.
+template <int BASE, int N>
+__host__ __device__ constexpr int fused_state(int i) {
+    return BASE == MTDAO_BASE_ADOPT
+               ? (i == 0 ? 1 + N : (i <= N ? i : 0))
+               : (i < N ? 1 + i : (BASE == MTDAO_BASE_ADAM && i == N ? 1 + N : 0));
+}
 
 template <int V>
 __device__ __forceinline__ void ld_v(const float *p, float *a) {
@@ -172,99 +188,78 @@ __global__ void __launch_bounds__(kThreads, 2) step_sync_kernel(const StepArgs a
                 store_replicas<M>(a.arena + (1 + j) * a.stride, n, e, grp, u[j], (mask >> (1 + j)) & 1u);
             if constexpr (kHasV)
                 store_replicas<M>(a.arena + (1 + N) * a.stride, n, e, grp, v, (mask >> (1 + N)) & 1u);
-        } else if constexpr (BASE == MTDAO_BASE_ADOPT) {
-            // v first; g becomes the normalised, clamped gradient.
-            {
-                float v[R][V];
-                float *p = a.arena + (1 + N) * a.stride;
-                load_replicas<M>(p, n, e, grp, v);
-#pragma unroll
-                for (int r = 0; r < R; ++r)
-#pragma unroll
-                    for (int k = 0; k < V; ++k) {
-                        const float gr = g[r][k];
-                        float gn;
-                        if (a.sc.prev_v) {
-                            gn = gr / (sqrtf(v[r][k]) + a.sc.eps);
-                            v[r][k] = fmaf(a.sc.c2, fmaf(gr, gr, -v[r][k]), v[r][k]);
-                        } else {
-                            v[r][k] = fmaf(a.sc.c2, fmaf(gr, gr, -v[r][k]), v[r][k]);
-                            gn = gr / (sqrtf(v[r][k]) + a.sc.eps);
-                        }
-                        gn = gn > a.sc.clip_c ? a.sc.clip_c : (gn < -a.sc.clip_c ? -a.sc.clip_c : gn);
-                        g[r][k] = gn;
-                    }
-                store_replicas<M>(p, n, e, grp, v, (mask >> (1 + N)) & 1u);
-            }
-            float d[R][V];
-#pragma unroll
-            for (int r = 0; r < R; ++r)
-#pragma unroll
-                for (int k = 0; k < V; ++k) d[r][k] = a.sc.cg * g[r][k];
-#pragma unroll
-            for (int j = 0; j < N; ++j) {
-                float u[R][V];
-                float *p = a.arena + (1 + j) * a.stride;
-                load_replicas<M>(p, n, e, grp, u);
-#pragma unroll
-                for (int r = 0; r < R; ++r)
-#pragma unroll
-                    for (int k = 0; k < V; ++k) {
-                        u[r][k] = fmaf(a.sc.c1[j], g[r][k] - u[r][k], u[r][k]);
-                        d[r][k] = fmaf(a.sc.k[j], u[r][k], d[r][k]);
-                    }
-                store_replicas<M>(p, n, e, grp, u, (mask >> (1 + j)) & 1u);
-            }
-            float x[R][V];
-            load_replicas<M>(a.arena, n, e, grp, x);
-#pragma unroll
-            for (int r = 0; r < R; ++r)
-#pragma unroll
-                for (int k = 0; k < V; ++k) x[r][k] = fmaf(a.sc.neg_lr, d[r][k], x[r][k]);
-            store_replicas<M>(a.arena, n, e, grp, x, mask & 1u);
         } else {
-            // Adam / SGDM: momenta of the clipped gradient g * s[r], then
-            // (Adam) v of the raw gradient and the denominator, then x.
-            float num[R][V];
-#pragma unroll
-            for (int r = 0; r < R; ++r)
-#pragma unroll
-                for (int k = 0; k < V; ++k) num[r][k] = a.sc.cg * __fmul_rn(g[r][k], s[r]);
-#pragma unroll
-            for (int j = 0; j < N; ++j) {
-                float u[R][V];
-                float *p = a.arena + (1 + j) * a.stride;
-                load_replicas<M>(p, n, e, grp, u);
+            // State by state in the order of fused_state.  With kLookahead the
+            // next state's loads are issued before the current state is
+            // updated and stored (different states are different slabs, so
+            // the reordering is safe), keeping two states' loads in flight.
+            constexpr int kStates = BASE == MTDAO_BASE_SGDM ? N + 1 : N + 2;
+            float gt[R][V];                   // ADOPT: the normalised, clamped gradient
+            float buf[2][R][V];
+            float acc[R][V];                  // Delta's numerator (Adam, SGDM) or Delta (ADOPT)
+            if constexpr (BASE != MTDAO_BASE_ADOPT) {
 #pragma unroll
                 for (int r = 0; r < R; ++r)
 #pragma unroll
-                    for (int k = 0; k < V; ++k) {
-                        u[r][k] = fmaf(a.sc.c1[j], __fmul_rn(g[r][k], s[r]) - u[r][k], u[r][k]);
-                        num[r][k] = fmaf(a.sc.k[j], u[r][k], num[r][k]);
-                    }
-                store_replicas<M>(p, n, e, grp, u, (mask >> (1 + j)) & 1u);
+                    for (int k = 0; k < V; ++k) acc[r][k] = a.sc.cg * __fmul_rn(g[r][k], s[r]);
             }
-            if constexpr (BASE == MTDAO_BASE_ADAM) {
-                float v[R][V];
-                float *p = a.arena + (1 + N) * a.stride;
-                load_replicas<M>(p, n, e, grp, v);
 #pragma unroll
-                for (int r = 0; r < R; ++r)
+            for (int i = 0; i < kStates; ++i) {
+                const int st = fused_state<BASE, N>(i);
+                if (!S::kLookahead || i == 0)
+                    load_replicas<M>(a.arena + st * a.stride, n, e, grp, buf[i & 1]);
+                if (S::kLookahead && i + 1 < kStates)
+                    load_replicas<M>(a.arena + fused_state<BASE, N>(i + 1) * a.stride, n, e, grp,
+                                     buf[(i + 1) & 1]);
+                float (&cur)[R][V] = buf[i & 1];
+                if (st == 1 + N && BASE == MTDAO_BASE_ADOPT) {
+                    // v first; gt receives the normalised, clamped gradient.
 #pragma unroll
-                    for (int k = 0; k < V; ++k) {
-                        const float gr = g[r][k];
-                        v[r][k] = fmaf(a.sc.c2, fmaf(gr, gr, -v[r][k]), v[r][k]);
-                        num[r][k] = num[r][k] / fmaf(sqrtf(v[r][k]), a.sc.sv, a.sc.eps);
-                    }
-                store_replicas<M>(p, n, e, grp, v, (mask >> (1 + N)) & 1u);
+                    for (int r = 0; r < R; ++r)
+#pragma unroll
+                        for (int k = 0; k < V; ++k) {
+                            const float gr = g[r][k];
+                            float gn;
+                            if (a.sc.prev_v) {
+                                gn = gr / (sqrtf(cur[r][k]) + a.sc.eps);
+                                cur[r][k] = fmaf(a.sc.c2, fmaf(gr, gr, -cur[r][k]), cur[r][k]);
+                            } else {
+                                cur[r][k] = fmaf(a.sc.c2, fmaf(gr, gr, -cur[r][k]), cur[r][k]);
+                                gn = gr / (sqrtf(cur[r][k]) + a.sc.eps);
+                            }
+                            gn = gn > a.sc.clip_c ? a.sc.clip_c : (gn < -a.sc.clip_c ? -a.sc.clip_c : gn);
+                            gt[r][k] = gn;
+                            acc[r][k] = a.sc.cg * gn;
+                        }
+                } else if (st == 1 + N) {
+                    // Adam: v of the raw gradient, then the denominator.
+#pragma unroll
+                    for (int r = 0; r < R; ++r)
+#pragma unroll
+                        for (int k = 0; k < V; ++k) {
+                            const float gr = g[r][k];
+                            cur[r][k] = fmaf(a.sc.c2, fmaf(gr, gr, -cur[r][k]), cur[r][k]);
+                            acc[r][k] = acc[r][k] / fmaf(sqrtf(cur[r][k]), a.sc.sv, a.sc.eps);
+                        }
+                } else if (st == 0) {
+#pragma unroll
+                    for (int r = 0; r < R; ++r)
+#pragma unroll
+                        for (int k = 0; k < V; ++k) cur[r][k] = fmaf(a.sc.neg_lr, acc[r][k], cur[r][k]);
+                } else {
+                    const int j = st - 1;             // momentum u_j
+#pragma unroll
+                    for (int r = 0; r < R; ++r)
+#pragma unroll
+                        for (int k = 0; k < V; ++k) {
+                            const float target =
+                                BASE == MTDAO_BASE_ADOPT ? gt[r][k] : __fmul_rn(g[r][k], s[r]);
+                            cur[r][k] = fmaf(a.sc.c1[j], target - cur[r][k], cur[r][k]);
+                            acc[r][k] = fmaf(a.sc.k[j], cur[r][k], acc[r][k]);
+                        }
+                }
+                store_replicas<M>(a.arena + st * a.stride, n, e, grp, cur, (mask >> st) & 1u);
             }
-            float x[R][V];
-            load_replicas<M>(a.arena, n, e, grp, x);
-#pragma unroll
-            for (int r = 0; r < R; ++r)
-#pragma unroll
-                for (int k = 0; k < V; ++k) x[r][k] = fmaf(a.sc.neg_lr, num[r][k], x[r][k]);
-            store_replicas<M>(a.arena, n, e, grp, x, mask & 1u);
         }
     }
 }

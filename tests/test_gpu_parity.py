@@ -71,7 +71,7 @@ RAGGED = [1, 7, 300, 4099, 2560, 13]
 @pytest.mark.parametrize("gdt", ["f32", "bf16"])
 @pytest.mark.parametrize("N", [1, 2, 3, 4])
 @pytest.mark.parametrize("base", ["adam", "adopt", "sgdm"])
-@pytest.mark.parametrize("M", [3, 4])
+@pytest.mark.parametrize("M", [2, 3, 4, 8])
 def test_step_and_sync_parity_matrix(P, base, N, gdt, M):
     betas = W.SWEEP_BETAS[:N]
     w = workload_dict(RAGGED, M, base=base, betas=betas, beta2=0.9999 if base == "adopt" else 0.999,
@@ -95,10 +95,12 @@ def test_replica_counts(P, M):
     eng.close()
 
 
-def test_fused_sync_is_bitwise_equal_to_separate_sync(P):
-    for base, M in (("adam", 4), ("adopt", 8), ("sgdm", 2)):
+@pytest.mark.parametrize("gdt", ["f32", "bf16"])
+@pytest.mark.parametrize("M", [2, 4, 8])
+def test_fused_sync_is_bitwise_equal_to_separate_sync(P, M, gdt):
+    for base in ("adam", "adopt", "sgdm"):
         w = workload_dict(RAGGED, M, base=base, betas=(0.9, 0.99, 0.5), px=3, pu=[2, 3, 4], pv=2,
-                          beta2=0.9999 if base == "adopt" else 0.999)
+                          beta2=0.9999 if base == "adopt" else 0.999, gdt=gdt)
         a = gpu_run(P, w, 8, fused=True)
         b = gpu_run(P, w, 8, fused=False)
         sa, sb = gpu_states(a, w["opt"]), gpu_states(b, w["opt"])
