@@ -155,6 +155,43 @@ int mtdao_plan_layout(const int64_t *tensor_numel, int32_t n_tensors,
  */
 int mtdao_due_mask(const mtdao_config *cfg, int64_t step, uint32_t *mask_out);
 
+/*
+ * Half-life of an EMA with decay rate beta (section 2.1):
+ * tau_0.5(beta) = ln 0.5 / ln beta, the number of steps after which a
+ * value's weight in u = beta u + (1 - beta) g has halved.  *tau_out gets
+ * tau for 0 < beta < 1 and 0 for beta = 0.  MTDAO_ERR_INVALID for beta
+ * outside [0, 1) or a NULL output.  No device access.
+ */
+int mtdao_half_life(double beta, double *tau_out);
+
+/*
+ * Half-life sync strategy (appendix on the wall-clock model, table of the
+ * modelled configurations): the parameters keep period_x and every state
+ * with a decay rate is averaged once per half-life of that rate, rounded to
+ * the nearest integer, but never more often than the parameters:
+ *   K_x = period_x,  K_j = max(K_x, round(tau_0.5(beta_{1,j}))),
+ *   K_v = max(K_x, round(tau_0.5(beta_2)))    (K_v untouched for SGDM).
+ * The table's caption speaks of the closest power of two, but its entries
+ * (69, 693 and 6931 for beta = 0.99, 0.999 and 0.9999; K_x = 32 for
+ * beta = 0.95, whose half-life is 13.5) are these rounded half-lives; the
+ * entries are what is implemented.  Only the period fields of *cfg change.
+ * MTDAO_ERR_INVALID for a NULL cfg, period_x < 0, or a decay rate outside
+ * [0, 1).  No device access.
+ */
+int mtdao_config_half_life_periods(mtdao_config *cfg, int64_t period_x);
+
+/*
+ * Communication of a configuration relative to DDP, which averages one
+ * d-element vector (the gradient) every step (section 2.3, the reduction
+ * factor stated after the algorithm's description): each state s is
+ * averaged once every K_s steps, so
+ *   *factor_out = (1/K_x + sum_j 1/K_j + 1/K_v)^-1
+ * (no v term for SGDM; a period of 0, never averaged, adds nothing;
+ * +infinity when nothing is ever averaged).  MTDAO_ERR_INVALID for a NULL
+ * argument or a negative period.  No device access.
+ */
+int mtdao_comm_reduction(const mtdao_config *cfg, double *factor_out);
+
 /* ------------------------------------------------------------------ lifecycle */
 
 /*

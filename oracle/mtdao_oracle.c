@@ -114,6 +114,56 @@ unsigned mto_due_after_step(const mto_cfg *c, long long t)
     return mask;
 }
 
+/*
+ * Half-life of the EMA u = beta u + (1 - beta) g (section 2.1): the number
+ * of steps after which a past value's weight beta^k has fallen to 1/2,
+ * tau = ln(0.5) / ln(beta).  A rate of 0 remembers nothing: 0.
+ */
+double mto_half_life(double beta)
+{
+    if (beta == 0.0)
+        return 0.0;
+    return log(0.5) / log(beta);
+}
+
+/*
+ * The half-life sync strategy of the wall-clock appendix (its table of the
+ * modelled configurations): parameters every K_x steps; each momentum and
+ * the second moment every round(half-life of its rate) steps, but not more
+ * often than the parameters.  The caption mentions powers of two, yet the
+ * printed periods are the rounded half-lives; those are what this follows.
+ */
+static long long half_life_period(double beta, long long period_x)
+{
+    long long k = (long long)floor(mto_half_life(beta) + 0.5);
+    return k < period_x ? period_x : k;
+}
+
+void mto_half_life_periods(mto_cfg *c, long long period_x)
+{
+    c->period_x = period_x;
+    for (int j = 0; j < c->n_mom; ++j)
+        c->period_u[j] = half_life_period(c->beta1[j], period_x);
+    if (c->base != MTO_SGDM)
+        c->period_v = half_life_period(c->beta2, period_x);
+}
+
+/*
+ * Communication relative to DDP (section 2.3): DDP averages one
+ * d-vector per step; here state s is averaged once per K_s steps, so the
+ * saving is 1 / (1/K_x + sum_j 1/K_j + 1/K_v).  Periods of 0 (never) add
+ * nothing; if no state is ever averaged the saving is infinite.
+ */
+double mto_comm_reduction(const mto_cfg *c)
+{
+    double per_step = 0.0;
+    if (c->period_x > 0) per_step += 1.0 / (double)c->period_x;
+    for (int j = 0; j < c->n_mom; ++j)
+        if (c->period_u[j] > 0) per_step += 1.0 / (double)c->period_u[j];
+    if (c->base != MTO_SGDM && c->period_v > 0) per_step += 1.0 / (double)c->period_v;
+    return per_step > 0.0 ? 1.0 / per_step : INFINITY;
+}
+
 /* E_m[s]: replace s^m by the equal-weight mean over the M workers. */
 void mto_mean_over_workers(int M, long long n, double *s)
 {

@@ -107,6 +107,12 @@ def _load():
             lib.mto_state_stats.restype = None
             lib.mto_pseudo_grad_stats.argtypes = [ctypes.c_int, ctypes.c_longlong, dp, dp, dp]
             lib.mto_pseudo_grad_stats.restype = None
+            lib.mto_half_life.argtypes = [ctypes.c_double]
+            lib.mto_half_life.restype = ctypes.c_double
+            lib.mto_half_life_periods.argtypes = [cp, ctypes.c_longlong]
+            lib.mto_half_life_periods.restype = None
+            lib.mto_comm_reduction.argtypes = [cp]
+            lib.mto_comm_reduction.restype = ctypes.c_double
             _lib = lib
     return _lib
 
@@ -242,3 +248,26 @@ def mean_over_workers(s: np.ndarray) -> np.ndarray:
     lib = _load()
     lib.mto_mean_over_workers(M, s.size // M, _ptr(s))
     return s
+
+
+def half_life(beta: float) -> float:
+    """tau_0.5(beta) = ln 0.5 / ln beta (section 2.1)."""
+    return float(_load().mto_half_life(float(beta)))
+
+
+def half_life_periods(cfg: dict, period_x: int) -> dict:
+    """The half-life sync strategy (see mto_half_life_periods): a copy of
+    cfg with period_x, period_u and period_v set."""
+    c = make_cfg(cfg)
+    _load().mto_half_life_periods(ctypes.byref(c), int(period_x))
+    out = dict(cfg)
+    out["period_x"] = int(c.period_x)
+    out["period_u"] = [int(c.period_u[j]) for j in range(int(cfg["n_mom"]))]
+    out["period_v"] = int(c.period_v)
+    return out
+
+
+def comm_reduction(cfg: dict) -> float:
+    """Communication saving over DDP (see mto_comm_reduction)."""
+    c = make_cfg(cfg)
+    return float(_load().mto_comm_reduction(ctypes.byref(c)))

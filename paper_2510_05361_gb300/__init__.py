@@ -72,6 +72,9 @@ def _load():
         "mtdao_num_states": (ctypes.c_int32, [cfgp]),
         "mtdao_plan_layout": (ctypes.c_int, [i64p, ctypes.c_int32, i64p, i64p]),
         "mtdao_due_mask": (ctypes.c_int, [cfgp, ctypes.c_int64, ctypes.POINTER(ctypes.c_uint32)]),
+        "mtdao_half_life": (ctypes.c_int, [ctypes.c_double, ctypes.POINTER(ctypes.c_double)]),
+        "mtdao_config_half_life_periods": (ctypes.c_int, [cfgp, ctypes.c_int64]),
+        "mtdao_comm_reduction": (ctypes.c_int, [cfgp, ctypes.POINTER(ctypes.c_double)]),
         "mtdao_create": (ctypes.c_int, [cfgp, ctypes.c_int32, i64p, ctypes.c_int32, ctypes.c_void_p,
                                         ctypes.POINTER(H)]),
         "mtdao_destroy": (None, [H]),
@@ -191,6 +194,24 @@ def mtdao_due_mask(cfg: mtdao_config, step: int) -> int:
     m = ctypes.c_uint32()
     _check(lib.mtdao_due_mask(ctypes.byref(cfg), int(step), ctypes.byref(m)))
     return int(m.value)
+
+
+def mtdao_half_life(beta: float) -> float:
+    tau = ctypes.c_double()
+    _check(lib.mtdao_half_life(float(beta), ctypes.byref(tau)))
+    return float(tau.value)
+
+
+def mtdao_config_half_life_periods(cfg: mtdao_config, period_x: int) -> mtdao_config:
+    """Sets cfg's periods in place (and returns cfg)."""
+    _check(lib.mtdao_config_half_life_periods(ctypes.byref(cfg), int(period_x)))
+    return cfg
+
+
+def mtdao_comm_reduction(cfg: mtdao_config) -> float:
+    f = ctypes.c_double()
+    _check(lib.mtdao_comm_reduction(ctypes.byref(cfg), ctypes.byref(f)))
+    return float(f.value)
 
 
 def mtdao_create(cfg: mtdao_config, M: int, numels, stream: int = 0):

@@ -6,6 +6,7 @@
 // where mtdao.h says it synchronises.
 #include <cuda_runtime.h>
 
+#include <algorithm>
 #include <cmath>
 #include <cstdarg>
 #include <cstdio>
@@ -335,6 +336,46 @@ extern "C" int mtdao_due_mask(const mtdao_config *cfg, int64_t step, uint32_t *m
     if (cfg == nullptr || mask_out == nullptr || step < 0)
         return set_error(nullptr, MTDAO_ERR_INVALID, "due_mask: bad arguments");
     *mask_out = due_mask(cfg, step);
+    return MTDAO_OK;
+}
+
+extern "C" int mtdao_half_life(double beta, double *tau_out) {
+    if (tau_out == nullptr || !(beta >= 0.0 && beta < 1.0))
+        return set_error(nullptr, MTDAO_ERR_INVALID, "half_life: beta must lie in [0, 1)");
+    *tau_out = beta == 0.0 ? 0.0 : std::log(0.5) / std::log(beta);
+    return MTDAO_OK;
+}
+
+extern "C" int mtdao_config_half_life_periods(mtdao_config *cfg, int64_t period_x) {
+    if (cfg == nullptr || period_x < 0 || cfg->n_mom < 1 || cfg->n_mom > MTDAO_MAX_MOM)
+        return set_error(nullptr, MTDAO_ERR_INVALID, "half_life_periods: bad arguments");
+    const bool has_v = cfg->base != MTDAO_BASE_SGDM;
+    int64_t k_u[MTDAO_MAX_MOM], k_v = cfg->period_v;
+    for (int j = 0; j <= cfg->n_mom; ++j) {
+        if (j == cfg->n_mom && !has_v) break;
+        const double beta = j < cfg->n_mom ? cfg->beta1[j] : cfg->beta2;
+        double tau;
+        if (mtdao_half_life(beta, &tau) != MTDAO_OK) return MTDAO_ERR_INVALID;
+        const int64_t k = std::max<int64_t>(period_x, std::llround(tau));
+        if (j < cfg->n_mom) k_u[j] = k; else k_v = k;
+    }
+    cfg->period_x = period_x;
+    for (int j = 0; j < cfg->n_mom; ++j) cfg->period_u[j] = k_u[j];
+    cfg->period_v = k_v;
+    return MTDAO_OK;
+}
+
+extern "C" int mtdao_comm_reduction(const mtdao_config *cfg, double *factor_out) {
+    if (cfg == nullptr || factor_out == nullptr || cfg->n_mom < 1 || cfg->n_mom > MTDAO_MAX_MOM)
+        return set_error(nullptr, MTDAO_ERR_INVALID, "comm_reduction: bad arguments");
+    const int n = cfg->n_mom + (cfg->base == MTDAO_BASE_SGDM ? 1 : 2);
+    double vectors_per_step = 0.0;
+    for (int s = 0; s < n; ++s) {
+        const int64_t k = s == 0 ? cfg->period_x : (s <= cfg->n_mom ? cfg->period_u[s - 1] : cfg->period_v);
+        if (k < 0) return set_error(nullptr, MTDAO_ERR_INVALID, "comm_reduction: negative period");
+        if (k > 0) vectors_per_step += 1.0 / static_cast<double>(k);
+    }
+    *factor_out = vectors_per_step > 0.0 ? 1.0 / vectors_per_step : HUGE_VAL;
     return MTDAO_OK;
 }
 

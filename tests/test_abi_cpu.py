@@ -125,3 +125,46 @@ def test_null_handle_is_safe(P):
     P.lib.mtdao_destroy(None)
     assert P.lib.mtdao_get_step(None) == -1
     assert P.lib.mtdao_sync(None, 1) == P.ERR_INVALID
+
+
+@pytest.mark.parametrize("base,betas,beta2,kx", [
+    ("adam", (0.95,), 0.99, 32), ("adopt", (0.95,), 0.9999, 32), ("adam", (0.999,), 0.999, 32),
+    ("adopt", (0.999,), 0.9999, 32), ("adam", (0.9, 0.999, 0.5), 0.999, 16),
+    ("sgdm", (0.99, 0.0), 0.999, 8), ("adopt", (0.9, 0.99), 0.9999, 0), ("adam", (0.9999,), 0.9, 1000),
+])
+def test_half_life_helpers_match_the_oracle(P, base, betas, beta2, kx):
+    """mtdao_half_life / mtdao_config_half_life_periods / mtdao_comm_reduction
+    against the oracle's own versions (which the pin suite ties to the
+    periods printed in the wall-clock appendix and to the sync count)."""
+    from oracle.oracle import comm_reduction, half_life, half_life_periods
+    for b in (*betas, beta2):
+        assert P.mtdao_half_life(b) == pytest.approx(half_life(b), rel=1e-15)
+    opt = _opt(base, betas, beta2=beta2, bias_correction=(base == "adam"))
+    cfg = P.mtdao_config_half_life_periods(P.make_config(opt), kx)
+    ref = half_life_periods(opt, kx)
+    assert cfg.period_x == ref["period_x"] == kx
+    assert [cfg.period_u[j] for j in range(len(betas))] == ref["period_u"]
+    if base != "sgdm":
+        assert cfg.period_v == ref["period_v"]
+    P.mtdao_config_validate(cfg, 4)
+    assert P.mtdao_comm_reduction(cfg) == pytest.approx(comm_reduction(ref), rel=1e-15)
+
+
+def test_half_life_helpers_reject_bad_arguments(P):
+    for beta in (1.0, -0.1, float("nan"), 2.0):
+        with pytest.raises(P.MTDAOError) as e:
+            P.mtdao_half_life(beta)
+        assert e.value.code == P.ERR_INVALID
+    cfg = P.make_config(_opt())
+    before = (cfg.period_x, cfg.period_u[0], cfg.period_v)
+    with pytest.raises(P.MTDAOError):
+        P.mtdao_config_half_life_periods(cfg, -1)
+    cfg.beta2 = 1.0
+    with pytest.raises(P.MTDAOError):
+        P.mtdao_config_half_life_periods(cfg, 32)
+    assert (cfg.period_x, cfg.period_u[0], cfg.period_v) == before      # unchanged on error
+    cfg = P.make_config(_opt(period_x=0, period_u=[0, 0], period_v=0))
+    assert P.mtdao_comm_reduction(cfg) == float("inf")
+    cfg.period_v = -3
+    with pytest.raises(P.MTDAOError):
+        P.mtdao_comm_reduction(cfg)

@@ -55,6 +55,11 @@ MUTATIONS = {
     "variance_over_M_minus_1": ("out[0] += (v - mean) * (v - mean) / (double)M;",
                                 "out[0] += (v - mean) * (v - mean) / (double)(M - 1);"),
     "dot_with_worker_instead_of_mean": ("out[2 + M + m] += v * mean;", "out[2 + M + m] += v * v;"),
+    "half_life_period_truncated": ("long long k = (long long)floor(mto_half_life(beta) + 0.5);",
+                                   "long long k = (long long)floor(mto_half_life(beta));"),
+    "half_life_period_not_floored_at_kx": ("return k < period_x ? period_x : k;", "return k;"),
+    "comm_reduction_without_v": ("if (c->base != MTO_SGDM && c->period_v > 0) per_step",
+                                 "if (0 && c->period_v > 0) per_step"),
     "global_pseudo_grad_without_anchor": ("double global = sum / (double)M - a[i];",
                                           "double global = sum / (double)M;"),
 }

@@ -14,7 +14,8 @@ import numpy as np
 import pytest
 import torch
 
-from oracle.oracle import Oracle, grad_norm, adopt_clip_bound
+from oracle.oracle import Oracle, adopt_clip_bound, comm_reduction, grad_norm, half_life, \
+    half_life_periods
 
 HERE = os.path.dirname(os.path.abspath(__file__))
 
@@ -142,6 +143,64 @@ def test_paper_printed_half_life():
     crossing = (k - 1) + (lo - math.log(0.5)) / (lo - hi)
     assert abs(crossing - float(row["printed"])) <= float(row["tol"])
 
+
+
+HALF_LIFE_ROWS = ["halflife_desloc_adam", "halflife_desloc_adopt", "halflife_mtdao_adam",
+                  "halflife_mtdao_adopt"]
+
+
+@pytest.mark.parametrize("name", HALF_LIFE_ROWS)
+def test_paper_printed_half_life_periods(name):
+    """The wall-clock appendix's Half-Life configurations: K_u1 and K_v from
+    beta_1, beta_2 and K_x = 32, as printed (exact)."""
+    row = _golden()[name]
+    base = "adopt" if float(row["beta2"]) == 0.9999 else "adam"
+    c = cfg(base, (float(row["beta1"]),), beta2=float(row["beta2"]), bias=base == "adam")
+    got = half_life_periods(c, int(row["K_x"]))
+    assert got["period_x"] == int(row["K_x"])
+    assert got["period_u"] == [int(row["K_u"])]
+    assert got["period_v"] == int(row["K_v"])
+
+
+@pytest.mark.parametrize("beta", [0.8, 0.9, 0.99, 0.999, 0.9999])
+def test_half_life_matches_the_ema_impulse_response(beta):
+    """tau_0.5 is where the EMA's memory of one value halves: the oracle's
+    own EMA (an SGDM momentum fed zeros after a unit value) is above 1/2
+    after floor(tau) steps and below it after ceil(tau) steps."""
+    tau = half_life(beta)
+    assert tau != math.floor(tau)
+    o = Oracle(cfg("sgdm", (beta,)), 1, 1)
+    o.u[0, 0, 0] = 1.0
+    for s in range(math.ceil(tau)):
+        if s == math.floor(tau):
+            assert o.u[0, 0, 0] > 0.5
+        o.step(s, 0.0, np.zeros((1, 1)))
+    assert o.u[0, 0, 0] < 0.5
+    assert half_life(0.0) == 0.0
+
+
+@pytest.mark.parametrize("base,periods", [("adam", (8, (4, 16), 2)), ("adopt", (64, (16,), 16)),
+                                          ("sgdm", (3, (5, 7, 2), 0)), ("adam", (0, (4,), 0)),
+                                          ("adam", (1, (1, 1), 1))])
+def test_comm_reduction_counts_the_averaged_vectors(base, periods):
+    """The saving over DDP (one d-vector per step) equals T divided by the
+    number of state vectors the schedule averages over T steps, T a common
+    multiple of the periods (counted from the oracle's own sync rule)."""
+    px, pu, pv = periods
+    c = cfg(base, tuple([0.9] * len(pu)), bias=False)
+    c.update(period_x=px, period_u=list(pu), period_v=pv)
+    T = 1
+    for k in (px, pv, *pu):
+        if k > 0:
+            T = T * k // math.gcd(T, k)
+    T *= 3
+    o = Oracle(c, 2, 1)
+    vectors = sum(bin(o.due_before_step(t)).count("1") for t in range(1, T + 1))
+    assert comm_reduction(c) == pytest.approx(T / vectors, rel=1e-14)
+    if periods == (1, (1, 1), 1):
+        assert comm_reduction(c) == pytest.approx(1.0 / 4)     # every state every step
+    none = cfg(base, (0.9,), bias=False)
+    assert comm_reduction(none) == math.inf
 
 # ------------------------------------------------------------- Adam pins
 
