@@ -15,35 +15,30 @@ namespace mtdao {
 
 // ---------------------------------------------------------------- fused step + sync
 
-// Layout of the fused kernel's work.  A lane holds its elements of R
-// replicas for every state it touches, so registers grow with R * V:
-//   M = 2 : one lane group, R = 2, V = 4 elements (128-bit accesses); the
-//           states are loaded, updated and stored one after another.
-//   M = 4 : one lane group, R = 4, V = 2 (64-bit accesses); every load of
-//           the chunk is issued before any arithmetic, as in step_kernel.
-//   M = 8 : two lane groups (half-warps), R = 4, V = 4, state by state with
-//           a lookahead: the next state's loads are issued before the
-//           current state is updated and stored, so two states' loads are
-//           in flight; lanes q and q + 16 hold the same elements, replicas
-//           0..3 and 4..7, and combine their parts of the average by
-//           shuffles.
-// Measured on the flat 2^27 sweep (GB/s of the fused step, Adam, f32):
-// issuing all loads first lifts M = 4 from ~6180 to ~6480 (the plain step's
-// level) but costs M = 2 (6650 -> 6500) and M = 8 (register spills); the
-// one-state lookahead lifts M = 8 from 6030-6065 to 6485-6727 (ADOPT with
-// bf16 gradients: 5439 -> 6089) and leaves M = 2 unchanged.
+// Layout of the fused kernel's work.  A lane holds V = 4 consecutive
+// elements (128-bit accesses) of R replicas:
+//   M = 2, 4 : one lane group, R = M;
+//   M = 8    : two lane groups (half-warps), R = 4: lanes q and q + 16 hold
+//              the same elements, replicas 0..3 and 4..7, and combine their
+//              parts of the average by shuffles.
+// The states are visited one after another (fused_state order); the next
+// state's loads are issued before the current state is updated and stored,
+// so two states' loads are in flight per lane within the 128-register cap.
+// Measured on the flat 2^27 sweep (GB/s of the fused step, Adam, f32): the
+// lookahead lifts M = 8 from 6030-6065 to 6485-6727 (ADOPT with bf16
+// gradients: 5439 -> 6089) and M = 4 from 6413-6556 (2 elements per lane,
+// every load of the chunk first, as in step_kernel) to 6582-6718; M = 2 is
+// the same with or without it.
 template <int M>
 struct FusedShape {
     static constexpr int G = M == 8 ? 2 : 1;      // lane groups per warp
     static constexpr int R = M / G;               // replicas per lane
-    static constexpr bool kPrefetch = M == 4;     // all loads of a chunk first
-    static constexpr int V = kPrefetch ? 2 : 4;   // elements per lane
+    static constexpr int V = 4;                   // elements per lane
     static constexpr int kLanes = 32 / G;         // lanes per group
     static constexpr int kChunk = kLanes * V;     // elements per warp iteration
-    static constexpr bool kLookahead = M == 8;    // state by state, next state's loads early
 };
 
-// Order in which the state-by-state shapes visit the states (arena index
+// Order in which the fused kernel visits the states (arena index
 // 0 = x, 1 + j = u_j, 1 + N = v): ADOPT takes v first (it normalises the
 // gradient), Adam takes v after the momenta (it divides their combination),
 // x comes last.
@@ -54,36 +49,8 @@ __host__ __device__ constexpr int fused_state(int i) {
                : (i < N ? 1 + i : (BASE == MTDAO_BASE_ADAM && i == N ? 1 + N : 0));
 }
 
-template <int V>
-__device__ __forceinline__ void ld_v(const float *p, float *a) {
-    if constexpr (V == 4) {
-        to_array(ld_state(p), a);
-    } else {
-        const float2 t = __ldcs(reinterpret_cast<const float2 *>(p));
-        a[0] = t.x; a[1] = t.y;
-    }
-}
-template <int V>
-__device__ __forceinline__ void st_v(float *p, const float *a) {
-    if constexpr (V == 4) {
-        st_state(p, from_array(a));
-    } else {
-        __stcs(reinterpret_cast<float2 *>(p), make_float2(a[0], a[1]));
-    }
-}
-template <int GDT, int V>
-__device__ __forceinline__ void ld_grad_v(const void *g, int64_t e, float *a) {
-    if constexpr (V == 4) {
-        to_array(ld_grad<GDT>(g, e), a);
-    } else if constexpr (GDT == MTDAO_F32) {
-        const float2 t = __ldcs(reinterpret_cast<const float2 *>(static_cast<const float *>(g) + e));
-        a[0] = t.x; a[1] = t.y;
-    } else {
-        const unsigned int w =
-            __ldcs(reinterpret_cast<const unsigned int *>(static_cast<const uint16_t *>(g) + e));
-        a[0] = __uint_as_float(w << 16); a[1] = __uint_as_float(w & 0xffff0000u);
-    }
-}
+__device__ __forceinline__ void ld_v(const float *p, float *a) { to_array(ld_state(p), a); }
+__device__ __forceinline__ void st_v(float *p, const float *a) { st_state(p, from_array(a)); }
 
 // Writes one state's R local values (for V elements) to the lane's replicas:
 // as they are, or -- when the state is due -- all replaced by the replica
@@ -119,11 +86,11 @@ __device__ __forceinline__ void store_replicas(float *state, int64_t n_padded, i
         }
 #pragma unroll
         for (int r = 0; r < S::R; ++r)
-            st_v<S::V>(state + (grp * S::R + r) * n_padded + e, mean);
+            st_v(state + (grp * S::R + r) * n_padded + e, mean);
     } else {
 #pragma unroll
         for (int r = 0; r < S::R; ++r)
-            st_v<S::V>(state + (grp * S::R + r) * n_padded + e, val[r]);
+            st_v(state + (grp * S::R + r) * n_padded + e, val[r]);
     }
 }
 
@@ -132,7 +99,7 @@ __device__ __forceinline__ void load_replicas(const float *state, int64_t n_padd
                                               float (&val)[FusedShape<M>::R][FusedShape<M>::V]) {
     using S = FusedShape<M>;
 #pragma unroll
-    for (int r = 0; r < S::R; ++r) ld_v<S::V>(state + (grp * S::R + r) * n_padded + e, val[r]);
+    for (int r = 0; r < S::R; ++r) ld_v(state + (grp * S::R + r) * n_padded + e, val[r]);
 }
 
 template <int BASE, int N, int GDT, bool CLIP, int M>
@@ -157,109 +124,78 @@ __global__ void __launch_bounds__(kThreads, 2) step_sync_kernel(const StepArgs a
         const int64_t e = c * S::kChunk + V * q;
         float g[R][V];
 #pragma unroll
-        for (int r = 0; r < R; ++r) ld_grad_v<GDT, V>(a.grads, (grp * R + r) * n + e, g[r]);
+        for (int r = 0; r < R; ++r) to_array(ld_grad<GDT>(a.grads, (grp * R + r) * n + e), g[r]);
 
-        if constexpr (S::kPrefetch) {
-            // Every load of the chunk is issued before any arithmetic (as in
-            // step_kernel), then the shared per-element update, then the
-            // stores with the due averages.
-            constexpr bool kHasV = BASE != MTDAO_BASE_SGDM;
-            float x[R][V], u[N][R][V], v[R][V];
-            load_replicas<M>(a.arena, n, e, grp, x);
-#pragma unroll
-            for (int j = 0; j < N; ++j) load_replicas<M>(a.arena + (1 + j) * a.stride, n, e, grp, u[j]);
-            if constexpr (kHasV) load_replicas<M>(a.arena + (1 + N) * a.stride, n, e, grp, v);
+        // State by state in the order of fused_state; the next state's
+        // loads are issued before the current state is updated and
+        // stored (different states are different slabs, so the
+        // reordering is safe), keeping two states' loads in flight.
+        constexpr int kStates = BASE == MTDAO_BASE_SGDM ? N + 1 : N + 2;
+        float gt[R][V];                   // ADOPT: the normalised, clamped gradient
+        float buf[2][R][V];
+        float acc[R][V];                  // Delta's numerator (Adam, SGDM) or Delta (ADOPT)
+        if constexpr (BASE != MTDAO_BASE_ADOPT) {
 #pragma unroll
             for (int r = 0; r < R; ++r)
 #pragma unroll
-                for (int k = 0; k < V; ++k) {
-                    float uk[N];
+                for (int k = 0; k < V; ++k) acc[r][k] = a.sc.cg * __fmul_rn(g[r][k], s[r]);
+        }
 #pragma unroll
-                    for (int j = 0; j < N; ++j) uk[j] = u[j][r][k];
-                    float vk = kHasV ? v[r][k] : 0.0f;
-                    update_element<BASE, N>(a.sc, g[r][k], s[r], x[r][k], uk, vk);
-#pragma unroll
-                    for (int j = 0; j < N; ++j) u[j][r][k] = uk[j];
-                    if constexpr (kHasV) v[r][k] = vk;
-                }
-            store_replicas<M>(a.arena, n, e, grp, x, mask & 1u);
-#pragma unroll
-            for (int j = 0; j < N; ++j)
-                store_replicas<M>(a.arena + (1 + j) * a.stride, n, e, grp, u[j], (mask >> (1 + j)) & 1u);
-            if constexpr (kHasV)
-                store_replicas<M>(a.arena + (1 + N) * a.stride, n, e, grp, v, (mask >> (1 + N)) & 1u);
-        } else {
-            // State by state in the order of fused_state.  With kLookahead the
-            // next state's loads are issued before the current state is
-            // updated and stored (different states are different slabs, so
-            // the reordering is safe), keeping two states' loads in flight.
-            constexpr int kStates = BASE == MTDAO_BASE_SGDM ? N + 1 : N + 2;
-            float gt[R][V];                   // ADOPT: the normalised, clamped gradient
-            float buf[2][R][V];
-            float acc[R][V];                  // Delta's numerator (Adam, SGDM) or Delta (ADOPT)
-            if constexpr (BASE != MTDAO_BASE_ADOPT) {
+        for (int i = 0; i < kStates; ++i) {
+            const int st = fused_state<BASE, N>(i);
+            if (i == 0)
+                load_replicas<M>(a.arena + st * a.stride, n, e, grp, buf[0]);
+            if (i + 1 < kStates)
+                load_replicas<M>(a.arena + fused_state<BASE, N>(i + 1) * a.stride, n, e, grp,
+                                 buf[(i + 1) & 1]);
+            float (&cur)[R][V] = buf[i & 1];
+            if (st == 1 + N && BASE == MTDAO_BASE_ADOPT) {
+                // v first; gt receives the normalised, clamped gradient.
 #pragma unroll
                 for (int r = 0; r < R; ++r)
 #pragma unroll
-                    for (int k = 0; k < V; ++k) acc[r][k] = a.sc.cg * __fmul_rn(g[r][k], s[r]);
-            }
-#pragma unroll
-            for (int i = 0; i < kStates; ++i) {
-                const int st = fused_state<BASE, N>(i);
-                if (!S::kLookahead || i == 0)
-                    load_replicas<M>(a.arena + st * a.stride, n, e, grp, buf[i & 1]);
-                if (S::kLookahead && i + 1 < kStates)
-                    load_replicas<M>(a.arena + fused_state<BASE, N>(i + 1) * a.stride, n, e, grp,
-                                     buf[(i + 1) & 1]);
-                float (&cur)[R][V] = buf[i & 1];
-                if (st == 1 + N && BASE == MTDAO_BASE_ADOPT) {
-                    // v first; gt receives the normalised, clamped gradient.
-#pragma unroll
-                    for (int r = 0; r < R; ++r)
-#pragma unroll
-                        for (int k = 0; k < V; ++k) {
-                            const float gr = g[r][k];
-                            float gn;
-                            if (a.sc.prev_v) {
-                                gn = gr / (sqrtf(cur[r][k]) + a.sc.eps);
-                                cur[r][k] = fmaf(a.sc.c2, fmaf(gr, gr, -cur[r][k]), cur[r][k]);
-                            } else {
-                                cur[r][k] = fmaf(a.sc.c2, fmaf(gr, gr, -cur[r][k]), cur[r][k]);
-                                gn = gr / (sqrtf(cur[r][k]) + a.sc.eps);
-                            }
-                            gn = gn > a.sc.clip_c ? a.sc.clip_c : (gn < -a.sc.clip_c ? -a.sc.clip_c : gn);
-                            gt[r][k] = gn;
-                            acc[r][k] = a.sc.cg * gn;
-                        }
-                } else if (st == 1 + N) {
-                    // Adam: v of the raw gradient, then the denominator.
-#pragma unroll
-                    for (int r = 0; r < R; ++r)
-#pragma unroll
-                        for (int k = 0; k < V; ++k) {
-                            const float gr = g[r][k];
+                    for (int k = 0; k < V; ++k) {
+                        const float gr = g[r][k];
+                        float gn;
+                        if (a.sc.prev_v) {
+                            gn = gr / (sqrtf(cur[r][k]) + a.sc.eps);
                             cur[r][k] = fmaf(a.sc.c2, fmaf(gr, gr, -cur[r][k]), cur[r][k]);
-                            acc[r][k] = acc[r][k] / fmaf(sqrtf(cur[r][k]), a.sc.sv, a.sc.eps);
+                        } else {
+                            cur[r][k] = fmaf(a.sc.c2, fmaf(gr, gr, -cur[r][k]), cur[r][k]);
+                            gn = gr / (sqrtf(cur[r][k]) + a.sc.eps);
                         }
-                } else if (st == 0) {
+                        gn = gn > a.sc.clip_c ? a.sc.clip_c : (gn < -a.sc.clip_c ? -a.sc.clip_c : gn);
+                        gt[r][k] = gn;
+                        acc[r][k] = a.sc.cg * gn;
+                    }
+            } else if (st == 1 + N) {
+                // Adam: v of the raw gradient, then the denominator.
 #pragma unroll
-                    for (int r = 0; r < R; ++r)
+                for (int r = 0; r < R; ++r)
 #pragma unroll
-                        for (int k = 0; k < V; ++k) cur[r][k] = fmaf(a.sc.neg_lr, acc[r][k], cur[r][k]);
-                } else {
-                    const int j = st - 1;             // momentum u_j
+                    for (int k = 0; k < V; ++k) {
+                        const float gr = g[r][k];
+                        cur[r][k] = fmaf(a.sc.c2, fmaf(gr, gr, -cur[r][k]), cur[r][k]);
+                        acc[r][k] = acc[r][k] / fmaf(sqrtf(cur[r][k]), a.sc.sv, a.sc.eps);
+                    }
+            } else if (st == 0) {
 #pragma unroll
-                    for (int r = 0; r < R; ++r)
+                for (int r = 0; r < R; ++r)
 #pragma unroll
-                        for (int k = 0; k < V; ++k) {
-                            const float target =
-                                BASE == MTDAO_BASE_ADOPT ? gt[r][k] : __fmul_rn(g[r][k], s[r]);
-                            cur[r][k] = fmaf(a.sc.c1[j], target - cur[r][k], cur[r][k]);
-                            acc[r][k] = fmaf(a.sc.k[j], cur[r][k], acc[r][k]);
-                        }
-                }
-                store_replicas<M>(a.arena + st * a.stride, n, e, grp, cur, (mask >> st) & 1u);
+                    for (int k = 0; k < V; ++k) cur[r][k] = fmaf(a.sc.neg_lr, acc[r][k], cur[r][k]);
+            } else {
+                const int j = st - 1;             // momentum u_j
+#pragma unroll
+                for (int r = 0; r < R; ++r)
+#pragma unroll
+                    for (int k = 0; k < V; ++k) {
+                        const float target =
+                            BASE == MTDAO_BASE_ADOPT ? gt[r][k] : __fmul_rn(g[r][k], s[r]);
+                        cur[r][k] = fmaf(a.sc.c1[j], target - cur[r][k], cur[r][k]);
+                        acc[r][k] = fmaf(a.sc.k[j], cur[r][k], acc[r][k]);
+                    }
             }
+            store_replicas<M>(a.arena + st * a.stride, n, e, grp, cur, (mask >> st) & 1u);
         }
     }
 }
