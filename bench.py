@@ -39,7 +39,9 @@ PEAKS_FILE = os.path.join(ROOT, "MEASURED_PEAKS.json")
 TRAFFIC_FILE = os.path.join(ROOT, "profiles", "step_kernel_traffic.txt")
 STEP_KERNEL_SRC = os.path.join(ROOT, "paper_2510_05361_gb300", "csrc", "step_kernels.cuh")
 FALLBACK_HBM_GBS = 6800.0
+NOMINAL_HBM_GBS = 7900.0    # vendor figure for GB300 HBM3e, for context beside the measured peak
 L2_BYTES = 129 * 2 ** 20
+SOLO_LAUNCHES = 20          # timed launches of each standalone kernel (after 2 untimed)
 
 
 def parse_args():
@@ -345,19 +347,25 @@ def run_ours(args):
     peak, peak_kind = hbm_peak()
     achieved = step_bytes / (step_ms / 1e3) / 1e9
 
+    def launches(fn, reps=SOLO_LAUNCHES, skip=2):
+        """Device times (ms) of `reps` launches of fn after `skip` untimed
+        ones, each bracketed by events on the launching stream."""
+        out = []
+        for i in range(skip + reps):
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            if flush is not None:
+                flush.fill_(1.0)
+            a.record(stream)
+            fn()
+            b.record(stream)
+            torch.cuda.synchronize()
+            if i >= skip:
+                out.append(a.elapsed_time(b))
+        return out
+
     # standalone replica-average kernel (all states), timed separately
-    sync_ms = []
     all_mask = (1 << n_states) - 1
-    for i in range(6):
-        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        if flush is not None:
-            flush.fill_(1.0)
-        a.record(stream)
-        P.mtdao_sync(eng.h, all_mask)
-        b.record(stream)
-        torch.cuda.synchronize()
-        if i >= 2:
-            sync_ms.append(a.elapsed_time(b))
+    sync_ms = launches(lambda: P.mtdao_sync(eng.h, all_mask))
     sync_bytes = W.bytes_per_sync(w, n_states)
     sync_gbs = sync_bytes / (statistics.median(sync_ms) / 1e3) / 1e9
 
@@ -365,32 +373,14 @@ def run_ours(args):
     stats_ms = []
     if M <= 8:
         stats_out = torch.empty((n_states, 2 + 2 * M), dtype=torch.float64, device="cuda")
-        for i in range(6):
-            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-            if flush is not None:
-                flush.fill_(1.0)
-            a.record(stream)
-            P.mtdao_sync_stats(eng.h, all_mask, stats_out.data_ptr())
-            b.record(stream)
-            torch.cuda.synchronize()
-            if i >= 2:
-                stats_ms.append(a.elapsed_time(b))
+        stats_ms = launches(lambda: P.mtdao_sync_stats(eng.h, all_mask, stats_out.data_ptr()))
 
     # pseudo-gradient diagnostics: a read-only pass over x and the anchor
     pg_ms = []
     if M <= 8:
         P.mtdao_track_anchor(eng.h, 1)
         pg_out = torch.empty((2 * M + 2,), dtype=torch.float64, device="cuda")
-        for i in range(6):
-            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-            if flush is not None:
-                flush.fill_(1.0)
-            a.record(stream)
-            P.mtdao_pseudo_grad_stats(eng.h, 0, pg_out.data_ptr())
-            b.record(stream)
-            torch.cuda.synchronize()
-            if i >= 2:
-                pg_ms.append(a.elapsed_time(b))
+        pg_ms = launches(lambda: P.mtdao_pseudo_grad_stats(eng.h, 0, pg_out.data_ptr()))
         P.mtdao_track_anchor(eng.h, 0)
     pg_bytes = (M + 1) * n * 4
 
@@ -445,18 +435,23 @@ def run_ours(args):
                    "inputs larger than L2 (%.0f GB resident)" % ((n_states * 4 + g_bytes) * M * n / 1e9)),
             "parallelism": "replicas only" if world == 1 else "independent replica set per GPU",
         },
-        "step_kernel": {"ms_mean": step_ms, "ms_min": min(plain), "bytes": step_bytes,
-                        "gbs": achieved, "params_per_s": M * n / (step_ms / 1e3)},
+        "step_kernel": {"ms_mean": step_ms, "ms_median": statistics.median(plain), "ms_min": min(plain),
+                        "launches": len(plain), "bytes": step_bytes,
+                        "gbs": achieved, "frac_of_nominal": achieved / NOMINAL_HBM_GBS,
+                        "params_per_s": M * n / (step_ms / 1e3),
+                        "model_params_per_s": n / (step_ms / 1e3)},
         "sync_step_kernel": {"ms_mean": statistics.mean(sync_steps),
                              "gbs": step_bytes / (statistics.mean(sync_steps) / 1e3) / 1e9,
                              "launches_per_round": len(sync_steps) // args.steps},
-        "sync_kernel": {"ms_median": statistics.median(sync_ms), "bytes": sync_bytes, "gbs": sync_gbs,
+        "sync_kernel": {"ms_median": statistics.median(sync_ms), "ms_min": min(sync_ms),
+                        "launches": len(sync_ms), "bytes": sync_bytes, "gbs": sync_gbs,
                         "frac": sync_gbs / peak, "states": n_states},
-        "sync_stats_kernel": ({"ms_median": statistics.median(stats_ms),
+        "sync_stats_kernel": ({"ms_median": statistics.median(stats_ms), "ms_min": min(stats_ms),
                                "gbs": sync_bytes / (statistics.median(stats_ms) / 1e3) / 1e9,
                                "frac": sync_bytes / (statistics.median(stats_ms) / 1e3) / 1e9 / peak}
                               if stats_ms else None),
-        "pseudo_grad_stats_kernel": ({"ms_median": statistics.median(pg_ms), "bytes": pg_bytes,
+        "pseudo_grad_stats_kernel": ({"ms_median": statistics.median(pg_ms), "ms_min": min(pg_ms),
+                                      "bytes": pg_bytes,
                                       "gbs": pg_bytes / (statistics.median(pg_ms) / 1e3) / 1e9}
                                      if pg_ms else None),
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",

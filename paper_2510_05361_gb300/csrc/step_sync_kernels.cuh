@@ -21,7 +21,7 @@ namespace mtdao {
 //   M = 8    : two lane groups (half-warps), R = 4: lanes q and q + 16 hold
 //              the same elements, replicas 0..3 and 4..7, and combine their
 //              parts of the average by shuffles.
-// The states are visited one after another (fused_state order); the next
+// The states are visited one after another (state_order); the next
 // state's loads are issued before the current state is updated and stored,
 // so two states' loads are in flight per lane within the 128-register cap.
 // Measured on the flat 2^27 sweep (GB/s of the fused step, Adam, f32): the
@@ -37,17 +37,6 @@ struct FusedShape {
     static constexpr int kLanes = 32 / G;         // lanes per group
     static constexpr int kChunk = kLanes * V;     // elements per warp iteration
 };
-
-// Order in which the fused kernel visits the states (arena index
-// 0 = x, 1 + j = u_j, 1 + N = v): ADOPT takes v first (it normalises the
-// gradient), Adam takes v after the momenta (it divides their combination),
-// x comes last.
-template <int BASE, int N>
-__host__ __device__ constexpr int fused_state(int i) {
-    return BASE == MTDAO_BASE_ADOPT
-               ? (i == 0 ? 1 + N : (i <= N ? i : 0))
-               : (i < N ? 1 + i : (BASE == MTDAO_BASE_ADAM && i == N ? 1 + N : 0));
-}
 
 __device__ __forceinline__ void ld_v(const float *p, float *a) { to_array(ld_state(p), a); }
 __device__ __forceinline__ void st_v(float *p, const float *a) { st_state(p, from_array(a)); }
@@ -126,11 +115,13 @@ __global__ void __launch_bounds__(kThreads, 2) step_sync_kernel(const StepArgs a
 #pragma unroll
         for (int r = 0; r < R; ++r) to_array(ld_grad<GDT>(a.grads, (grp * R + r) * n + e), g[r]);
 
-        // State by state in the order of fused_state; the next state's
-        // loads are issued before the current state is updated and
-        // stored (different states are different slabs, so the
-        // reordering is safe), keeping two states' loads in flight.
-        constexpr int kStates = BASE == MTDAO_BASE_SGDM ? N + 1 : N + 2;
+        // State by state in state_order; the next state's loads are issued
+        // before the current state is updated and stored (different states
+        // are different slabs, so the reordering is safe).  The arithmetic
+        // is update_state's, written out per state (the same expressions,
+        // so the same bits; the written-out form keeps the M = 8 ADOPT
+        // instance within its registers).
+        constexpr int kStates = kNumStates<BASE, N>;
         float gt[R][V];                   // ADOPT: the normalised, clamped gradient
         float buf[2][R][V];
         float acc[R][V];                  // Delta's numerator (Adam, SGDM) or Delta (ADOPT)
@@ -142,11 +133,11 @@ __global__ void __launch_bounds__(kThreads, 2) step_sync_kernel(const StepArgs a
         }
 #pragma unroll
         for (int i = 0; i < kStates; ++i) {
-            const int st = fused_state<BASE, N>(i);
+            const int st = state_order<BASE, N>(i);
             if (i == 0)
                 load_replicas<M>(a.arena + st * a.stride, n, e, grp, buf[0]);
             if (i + 1 < kStates)
-                load_replicas<M>(a.arena + fused_state<BASE, N>(i + 1) * a.stride, n, e, grp,
+                load_replicas<M>(a.arena + state_order<BASE, N>(i + 1) * a.stride, n, e, grp,
                                  buf[(i + 1) & 1]);
             float (&cur)[R][V] = buf[i & 1];
             if (st == 1 + N && BASE == MTDAO_BASE_ADOPT) {
