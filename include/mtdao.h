@@ -345,6 +345,19 @@ int mtdao_grad_sqnorm(mtdao_handle h, const void *grads_dev, int32_t grad_dtype,
                       double *out_dev);
 
 /*
+ * Gradient health check (the paper has no counterpart; NaN and Inf
+ * gradients otherwise propagate into every state of the replica, as the
+ * algorithms written out would propagate them): out_dev (device, M doubles,
+ * caller-owned) receives the number of NaN or +-Inf values in replica m's
+ * gradient, exact.  A caller can skip a step whose count is nonzero (e.g.
+ * an overflow of bf16 gradients).  Same grid, workspace and
+ * determinism as mtdao_grad_sqnorm; reads the gradient once (g_b bytes per
+ * element).  Errors as mtdao_grad_sqnorm.
+ */
+int mtdao_grad_nonfinite(mtdao_handle h, const void *grads_dev, int32_t grad_dtype,
+                         double *out_dev);
+
+/*
  * mtdao_grad_sqnorm_static -- the per-replica sum of squares of
  * mtdao_grad_sqnorm for callers that cannot allocate device memory.
  * The paper has no counterpart; this is a library convenience.

@@ -92,6 +92,7 @@ def _load():
         "mtdao_track_anchor": (ctypes.c_int, [H, ctypes.c_uint32]),
         "mtdao_pseudo_grad_stats": (ctypes.c_int, [H, ctypes.c_int32, ctypes.c_void_p]),
         "mtdao_grad_sqnorm": (ctypes.c_int, [H, ctypes.c_void_p, ctypes.c_int32, ctypes.c_void_p]),
+        "mtdao_grad_nonfinite": (ctypes.c_int, [H, ctypes.c_void_p, ctypes.c_int32, ctypes.c_void_p]),
         "mtdao_grad_sqnorm_static": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_int32, ctypes.c_int32,
                                                     ctypes.c_int64, ctypes.c_void_p, ctypes.c_void_p]),
         "mtdao_get_state_ptr": (ctypes.c_int, [H, ctypes.c_int32, ctypes.c_int32,
@@ -274,6 +275,11 @@ def mtdao_sync_due(h) -> int:
 def mtdao_grad_sqnorm(h, grads_dev_ptr: int, grad_dtype: int, out_dev_ptr: int) -> None:
     _check(lib.mtdao_grad_sqnorm(h, ctypes.c_void_p(grads_dev_ptr), grad_dtype,
                                  ctypes.c_void_p(out_dev_ptr)), h)
+
+
+def mtdao_grad_nonfinite(h, grads_dev_ptr: int, grad_dtype: int, out_dev_ptr: int) -> None:
+    _check(lib.mtdao_grad_nonfinite(h, ctypes.c_void_p(grads_dev_ptr), grad_dtype,
+                                    ctypes.c_void_p(out_dev_ptr)), h)
 
 
 def mtdao_grad_sqnorm_static(grads_dev_ptr: int, grad_dtype: int, M: int, n_padded: int,

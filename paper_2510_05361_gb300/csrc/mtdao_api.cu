@@ -15,6 +15,8 @@
 #include <string>
 #include <vector>
 
+#include <nvtx3/nvToolsExt.h>
+
 #include "mtdao.h"
 #include "mtdao_internal.h"
 
@@ -92,6 +94,16 @@ struct mtdao_ctx {
 };
 
 namespace {
+
+// A named range around each entry point that enqueues GPU work, for Nsight
+// tools (ncu --nvtx --nvtx-include "mtdao_step/"); without a tool attached
+// a push/pop costs a few nanoseconds.
+struct Range {
+    explicit Range(const char *name) { nvtxRangePushA(name); }
+    ~Range() { nvtxRangePop(); }
+    Range(const Range &) = delete;
+    Range &operator=(const Range &) = delete;
+};
 
 thread_local std::string g_err;
 
@@ -525,6 +537,7 @@ static int enqueue_sync(mtdao_ctx *h, uint32_t mask) {
 
 extern "C" int mtdao_step(mtdao_handle h, const void *grads_dev, int32_t grad_dtype, double lr,
                           uint32_t sync_mask) {
+    Range range("mtdao_step");
     if (int rc = check_handle(h)) return rc;
     if (grads_dev == nullptr) return set_error(h, MTDAO_ERR_INVALID, "grads is NULL");
     if (!aligned16(grads_dev)) return set_error(h, MTDAO_ERR_ALIGN, "grads not 16-byte aligned");
@@ -575,6 +588,7 @@ extern "C" int mtdao_step(mtdao_handle h, const void *grads_dev, int32_t grad_dt
 
 extern "C" int mtdao_run(mtdao_handle h, const void *grads_dev, int64_t grads_stride_bytes,
                          int32_t grad_dtype, const double *lrs, int32_t count) {
+    Range range("mtdao_run");
     if (int rc = check_handle(h)) return rc;
     if (count < 0 || (count > 0 && (grads_dev == nullptr || lrs == nullptr)))
         return set_error(h, MTDAO_ERR_INVALID, "run: bad count or NULL arguments");
@@ -589,6 +603,7 @@ extern "C" int mtdao_run(mtdao_handle h, const void *grads_dev, int64_t grads_st
 
 extern "C" int mtdao_step_host(mtdao_handle h, const void *grads_host, int32_t grad_dtype, double lr,
                                uint32_t sync_mask) {
+    Range range("mtdao_step_host");
     if (int rc = check_handle(h)) return rc;
     if (grads_host == nullptr) return set_error(h, MTDAO_ERR_INVALID, "grads is NULL");
     if (grad_dtype != MTDAO_F32 && grad_dtype != MTDAO_BF16)
@@ -638,6 +653,7 @@ extern "C" int mtdao_step_host(mtdao_handle h, const void *grads_host, int32_t g
 }
 
 extern "C" int mtdao_sync(mtdao_handle h, uint32_t mask) {
+    Range range("mtdao_sync");
     if (int rc = check_handle(h)) return rc;
     if (mask >> h->n_states) return set_error(h, MTDAO_ERR_INVALID, "sync mask 0x%x has bits beyond "
                                               "the %d states", mask, h->n_states);
@@ -649,6 +665,7 @@ extern "C" int mtdao_sync(mtdao_handle h, uint32_t mask) {
 }
 
 extern "C" int mtdao_sync_stats(mtdao_handle h, uint32_t mask, double *stats_dev) {
+    Range range("mtdao_sync_stats");
     if (int rc = check_handle(h)) return rc;
     if (stats_dev == nullptr) return set_error(h, MTDAO_ERR_INVALID, "stats is NULL");
     if (mask >> h->n_states) return set_error(h, MTDAO_ERR_INVALID, "sync mask 0x%x has bits beyond "
@@ -702,6 +719,7 @@ extern "C" int mtdao_track_anchor(mtdao_handle h, uint32_t state_mask) {
 }
 
 extern "C" int mtdao_pseudo_grad_stats(mtdao_handle h, int32_t state, double *out_dev) {
+    Range range("mtdao_pseudo_grad_stats");
     if (int rc = check_handle(h)) return rc;
     if (out_dev == nullptr) return set_error(h, MTDAO_ERR_INVALID, "out is NULL");
     if (state < 0 || state >= h->n_states) return set_error(h, MTDAO_ERR_INVALID, "state %d out of range", state);
@@ -724,8 +742,25 @@ extern "C" int mtdao_sync_due(mtdao_handle h, uint32_t *mask_out) {
     return MTDAO_OK;
 }
 
+extern "C" int mtdao_grad_nonfinite(mtdao_handle h, const void *grads_dev, int32_t grad_dtype,
+                                    double *out_dev) {
+    Range range("mtdao_grad_nonfinite");
+    if (int rc = check_handle(h)) return rc;
+    if (grads_dev == nullptr || out_dev == nullptr)
+        return set_error(h, MTDAO_ERR_INVALID, "grads or out is NULL");
+    if (!aligned16(grads_dev)) return set_error(h, MTDAO_ERR_ALIGN, "grads not 16-byte aligned");
+    if (grad_dtype != MTDAO_F32 && grad_dtype != MTDAO_BF16)
+        return set_error(h, MTDAO_ERR_INVALID, "unknown gradient dtype %d", grad_dtype);
+    if (int rc = select_device(h)) return rc;
+    cudaError_t e = launch_grad_nonfinite(grads_dev, grad_dtype, h->M, h->n_padded, h->norm_blocks,
+                                          h->norm_partial, out_dev, h->stream);
+    if (e != cudaSuccess) return cuda_fail(h, e, "non-finite count launch");
+    return MTDAO_OK;
+}
+
 extern "C" int mtdao_grad_sqnorm(mtdao_handle h, const void *grads_dev, int32_t grad_dtype,
                                  double *out_dev) {
+    Range range("mtdao_grad_sqnorm");
     if (int rc = check_handle(h)) return rc;
     if (grads_dev == nullptr || out_dev == nullptr)
         return set_error(h, MTDAO_ERR_INVALID, "grads or out is NULL");

@@ -81,6 +81,11 @@ cudaError_t launch_grad_sqnorm(const void *grads, int grad_dtype, int32_t M, int
                                int blocks_per_replica, double *partial, double *out,
                                float *clip_scale, double rho, cudaStream_t stream);
 
+// Number of NaN / +-Inf gradient values per replica into out[m] (double,
+// exact), with the grid and workspace of launch_grad_sqnorm.
+cudaError_t launch_grad_nonfinite(const void *grads, int grad_dtype, int32_t M, int64_t n_padded,
+                                  int blocks_per_replica, double *partial, double *out, cudaStream_t stream);
+
 // Pseudo-gradient diagnostics of x[M][n] against anchor[n] into stats[2M+2]
 // (as documented for mtdao_pseudo_grad_stats); M must be 1..8.  Uses the
 // sync-diagnostics workspace.

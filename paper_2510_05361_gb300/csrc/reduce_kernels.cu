@@ -115,6 +115,27 @@ __global__ void __launch_bounds__(kNormThreads) sqnorm_partial_kernel(const void
     if (threadIdx.x == 0) partial[static_cast<int64_t>(m) * nb + blockIdx.x] = total;
 }
 
+// Number of NaN or +-Inf values (all exponent bits set) per replica, with
+// the same fixed grid and reduction order as the sum of squares; counts are
+// integers well below 2^53, so the double partials are exact.
+template <int GDT>
+__global__ void __launch_bounds__(kNormThreads) nonfinite_partial_kernel(const void *g, int64_t n,
+                                                                         double *partial) {
+    const int m = blockIdx.y;
+    const int nb = gridDim.x;
+    const int64_t nv = n / 4;
+    uint64_t count = 0;
+    for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < nv;
+         i += static_cast<int64_t>(nb) * blockDim.x) {
+        const float4 q = ld_grad<GDT>(g, m * n + 4 * i);
+        const uint32_t e = 0x7f800000u;
+        count += ((__float_as_uint(q.x) & e) == e) + ((__float_as_uint(q.y) & e) == e) +
+                 ((__float_as_uint(q.z) & e) == e) + ((__float_as_uint(q.w) & e) == e);
+    }
+    const double total = block_sum(static_cast<double>(count));
+    if (threadIdx.x == 0) partial[static_cast<int64_t>(m) * nb + blockIdx.x] = total;
+}
+
 __global__ void __launch_bounds__(kNormThreads) sqnorm_finalize_kernel(const double *partial, int nb,
                                                                        double *out, float *clip_scale,
                                                                        double rho) {
@@ -368,6 +389,19 @@ cudaError_t launch_sync(const SyncArgs &a, int num_sms, cudaStream_t stream) {
 int norm_blocks_per_replica(int num_sms, int M) {
     int b = (4 * num_sms) / (M > 0 ? M : 1);
     return b < 1 ? 1 : b;
+}
+
+cudaError_t launch_grad_nonfinite(const void *grads, int grad_dtype, int32_t M, int64_t n_padded,
+                                  int blocks_per_replica, double *partial, double *out, cudaStream_t stream) {
+    dim3 grid(static_cast<unsigned>(blocks_per_replica), static_cast<unsigned>(M));
+    if (grad_dtype == MTDAO_F32)
+        nonfinite_partial_kernel<MTDAO_F32><<<grid, kNormThreads, 0, stream>>>(grads, n_padded, partial);
+    else
+        nonfinite_partial_kernel<MTDAO_BF16><<<grid, kNormThreads, 0, stream>>>(grads, n_padded, partial);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    sqnorm_finalize_kernel<<<M, kNormThreads, 0, stream>>>(partial, blocks_per_replica, out, nullptr, 0.0);
+    return cudaGetLastError();
 }
 
 cudaError_t launch_grad_sqnorm(const void *grads, int grad_dtype, int32_t M, int64_t n_padded,

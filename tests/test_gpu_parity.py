@@ -140,6 +140,38 @@ def test_grad_sqnorm(P, gdt):
     eng.close()
 
 
+@pytest.mark.parametrize("gdt", ["f32", "bf16"])
+def test_grad_nonfinite_counts(P, gdt):
+    """mtdao_grad_nonfinite counts exactly the NaN / +-Inf values planted in
+    each replica's gradient (counts known by construction); the largest
+    finite values, subnormals and -0 are not counted."""
+    M = 5
+    w = workload_dict(RAGGED + [70000], M, gdt=gdt)
+    lay = W.layout(w["shapes"])
+    n = lay["n_padded"]
+    g = host_grads(w, lay, SEED_G, 0, np.arange(n))
+    rng = np.random.default_rng(31)
+    extremes = {(0, 1): 3.0e38, (1, 2): -3.0e38, (2, 3): 1e-45, (3, 4): -0.0, (4, 5): 1e-39}
+    for (m, i), v in extremes.items():
+        g[m, i] = np.float32(v)
+    expected = []
+    for m in range(M):
+        k = [0, 1, 7, 300, 4099][m]
+        pos = rng.choice(np.arange(8, n), size=k, replace=False)
+        g[m, pos] = rng.choice(np.array([np.nan, np.inf, -np.inf], np.float32), size=k)
+        expected.append(float(k))
+    gd = to_dev(g, gdt)
+    dt = P.BF16 if gdt == "bf16" else P.F32
+    eng = P.MTDAO(w["opt"], M, w["shapes"])
+    out = torch.full((M,), -1.0, dtype=torch.float64, device="cuda")
+    P.mtdao_grad_nonfinite(eng.h, gd.data_ptr(), dt, out.data_ptr())
+    assert out.cpu().numpy().tolist() == expected
+    clean = to_dev(host_grads(w, lay, SEED_G, 1, np.arange(n)), gdt)
+    P.mtdao_grad_nonfinite(eng.h, clean.data_ptr(), dt, out.data_ptr())
+    assert out.cpu().numpy().tolist() == [0.0] * M
+    eng.close()
+
+
 @pytest.mark.parametrize("clip", ["elementwise", "none"])
 def test_adopt_clip_parity(P, clip):
     w = workload_dict(RAGGED, 4, base="adopt", betas=(0.95, 0.999), beta2=0.9999, clip=clip,
