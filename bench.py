@@ -384,6 +384,13 @@ def run_ours(args):
         P.mtdao_track_anchor(eng.h, 0)
     pg_bytes = (M + 1) * n * 4
 
+    # S0: per-replica gradient sum of squares (the clip(g, rho) pre-pass) and
+    # the non-finite count, each one read of the resident gradients
+    norm_out = torch.empty((M,), dtype=torch.float64, device="cuda")
+    norm_ms = launches(lambda: P.mtdao_grad_sqnorm(eng.h, grads.data_ptr(), gdt, norm_out.data_ptr()))
+    nonfinite_ms = launches(lambda: P.mtdao_grad_nonfinite(eng.h, grads.data_ptr(), gdt, norm_out.data_ptr()))
+    grad_bytes = M * n * g_bytes
+
     # end to end through the host-buffer C-ABI call
     e2e = None
     if not args.no_e2e and args.e2e_rounds > 0:
@@ -454,6 +461,12 @@ def run_ours(args):
                                       "bytes": pg_bytes,
                                       "gbs": pg_bytes / (statistics.median(pg_ms) / 1e3) / 1e9}
                                      if pg_ms else None),
+        "grad_sqnorm_kernel": {"ms_median": statistics.median(norm_ms), "ms_min": min(norm_ms),
+                               "bytes": grad_bytes,
+                               "gbs": grad_bytes / (statistics.median(norm_ms) / 1e3) / 1e9,
+                               "frac": grad_bytes / (statistics.median(norm_ms) / 1e3) / 1e9 / peak},
+        "grad_nonfinite_kernel": {"ms_median": statistics.median(nonfinite_ms), "bytes": grad_bytes,
+                                  "gbs": grad_bytes / (statistics.median(nonfinite_ms) / 1e3) / 1e9},
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                      "frac": achieved / peak, "traffic": traffic, "peak_kind": peak_kind,
                      "kernel": step_kernel_name(opt, w["grad_dtype"])},

@@ -14,6 +14,7 @@
 #include <cuda_runtime.h>
 #include <cmath>
 #include <cstdint>
+#include <type_traits>
 
 #include "mtdao_internal.h"
 #include "replica_mean.cuh"
@@ -96,20 +97,59 @@ __device__ double block_sum(double v) {
     return total;
 }
 
+// Positions (groups of 4 elements) a thread of the norm kernels loads
+// before it accumulates them: i, i + T, ..., i + (U - 1) T with T the
+// replica's thread count, the same order as a plain grid-stride loop, so
+// the sums do not depend on the unrolling.  64 bytes per thread in flight:
+// 4 positions of f32, 8 of bf16.
 template <int GDT>
-__global__ void __launch_bounds__(kNormThreads) sqnorm_partial_kernel(const void *g, int64_t n,
+constexpr int kNormUnroll = GDT == MTDAO_F32 ? 4 : 8;
+
+// Four gradient values as loaded (f32: float4; bf16: two packed words, 2
+// registers instead of 4 until they are widened) and their fp32 values.
+template <int GDT>
+using GradWords = typename std::conditional<GDT == MTDAO_F32, float4, uint2>::type;
+
+template <int GDT>
+__device__ __forceinline__ GradWords<GDT> ld_grad_words(const void *g, int64_t e) {
+    if constexpr (GDT == MTDAO_F32)
+        return __ldcs(reinterpret_cast<const float4 *>(static_cast<const float *>(g) + e));
+    else
+        return __ldcs(reinterpret_cast<const uint2 *>(static_cast<const uint16_t *>(g) + e));
+}
+
+template <int GDT>
+__device__ __forceinline__ float4 widen(GradWords<GDT> w) {
+    if constexpr (GDT == MTDAO_F32)
+        return w;
+    else
+        return make_float4(__uint_as_float(w.x << 16), __uint_as_float(w.x & 0xffff0000u),
+                           __uint_as_float(w.y << 16), __uint_as_float(w.y & 0xffff0000u));
+}
+
+template <int GDT>
+__global__ void __launch_bounds__(kNormThreads, 4) sqnorm_partial_kernel(const void *g, int64_t n,
                                                                       double *partial) {
     const int m = blockIdx.y;
     const int nb = gridDim.x;
     const int64_t nv = n / 4;
+    const int64_t T = static_cast<int64_t>(nb) * blockDim.x;
     float sum = 0.0f, comp = 0.0f;
     for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < nv;
-         i += static_cast<int64_t>(nb) * blockDim.x) {
-        const float4 q = ld_grad<GDT>(g, m * n + 4 * i);
-        const float y = fmaf(q.x, q.x, fmaf(q.y, q.y, fmaf(q.z, q.z, __fmul_rn(q.w, q.w)))) - comp;
-        const float t = sum + y;
-        comp = (t - sum) - y;
-        sum = t;
+         i += kNormUnroll<GDT> * T) {
+        GradWords<GDT> w[kNormUnroll<GDT>];
+#pragma unroll
+        for (int u = 0; u < kNormUnroll<GDT>; ++u)
+            if (i + u * T < nv) w[u] = ld_grad_words<GDT>(g, m * n + 4 * (i + u * T));
+#pragma unroll
+        for (int u = 0; u < kNormUnroll<GDT>; ++u) {
+            if (i + u * T >= nv) break;
+            const float4 q = widen<GDT>(w[u]);
+            const float y = fmaf(q.x, q.x, fmaf(q.y, q.y, fmaf(q.z, q.z, __fmul_rn(q.w, q.w)))) - comp;
+            const float t = sum + y;
+            comp = (t - sum) - y;
+            sum = t;
+        }
     }
     const double total = block_sum(static_cast<double>(sum) - static_cast<double>(comp));
     if (threadIdx.x == 0) partial[static_cast<int64_t>(m) * nb + blockIdx.x] = total;
@@ -119,18 +159,27 @@ __global__ void __launch_bounds__(kNormThreads) sqnorm_partial_kernel(const void
 // the same fixed grid and reduction order as the sum of squares; counts are
 // integers well below 2^53, so the double partials are exact.
 template <int GDT>
-__global__ void __launch_bounds__(kNormThreads) nonfinite_partial_kernel(const void *g, int64_t n,
+__global__ void __launch_bounds__(kNormThreads, 4) nonfinite_partial_kernel(const void *g, int64_t n,
                                                                          double *partial) {
     const int m = blockIdx.y;
     const int nb = gridDim.x;
     const int64_t nv = n / 4;
-    uint64_t count = 0;
+    const int64_t T = static_cast<int64_t>(nb) * blockDim.x;
+    const uint32_t e = 0x7f800000u;
+    uint32_t count = 0;                // at most 4 nv / T per thread
     for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < nv;
-         i += static_cast<int64_t>(nb) * blockDim.x) {
-        const float4 q = ld_grad<GDT>(g, m * n + 4 * i);
-        const uint32_t e = 0x7f800000u;
-        count += ((__float_as_uint(q.x) & e) == e) + ((__float_as_uint(q.y) & e) == e) +
-                 ((__float_as_uint(q.z) & e) == e) + ((__float_as_uint(q.w) & e) == e);
+         i += kNormUnroll<GDT> * T) {
+        GradWords<GDT> w[kNormUnroll<GDT>];
+#pragma unroll
+        for (int u = 0; u < kNormUnroll<GDT>; ++u)
+            if (i + u * T < nv) w[u] = ld_grad_words<GDT>(g, m * n + 4 * (i + u * T));
+#pragma unroll
+        for (int u = 0; u < kNormUnroll<GDT>; ++u) {
+            if (i + u * T >= nv) break;
+            const float4 q = widen<GDT>(w[u]);
+            count += ((__float_as_uint(q.x) & e) == e) + ((__float_as_uint(q.y) & e) == e) +
+                     ((__float_as_uint(q.z) & e) == e) + ((__float_as_uint(q.w) & e) == e);
+        }
     }
     const double total = block_sum(static_cast<double>(count));
     if (threadIdx.x == 0) partial[static_cast<int64_t>(m) * nb + blockIdx.x] = total;

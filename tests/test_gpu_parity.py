@@ -385,6 +385,37 @@ def test_zero_size_and_single_element_tensors(P):
         eng.close()
 
 
+@pytest.mark.parametrize("base,M", [("adam", 4), ("adopt", 8), ("sgdm", 2), ("adam", 3)])
+def test_padding_canaries_are_untouched(P, base, M):
+    """Canary values planted in the parameters' alignment padding (between
+    tensors and at the end) survive steps, fused and standalone averages bit
+    for bit, u and v stay zero there, and the tensors' own elements are
+    bit-identical to a run without canaries: no kernel reads or writes
+    across a tensor boundary."""
+    w = workload_dict(RAGGED, M, base=base, betas=(0.9, 0.99), px=3, pu=[2, 4], pv=2,
+                      beta2=0.9999 if base == "adopt" else 0.999)
+    lay = W.layout(w["shapes"])
+    n = lay["n_padded"]
+    inside = G.in_tensor_mask(np.arange(n), lay["offsets"], lay["numels"])
+    assert (~inside).sum() > 0
+    x0 = G.init_params(w, lay, SEED_I, np.arange(n))
+    x0c = x0.copy()
+    x0c[~inside] = np.float32(1234.5)
+    runs = []
+    for start in (x0, x0c):
+        eng = gpu_run(P, w, 9, x0=start)
+        eng.sync(0b1)                                     # one standalone average too
+        torch.cuda.synchronize()
+        runs.append(gpu_states(eng, w["opt"]))
+        eng.close()
+    plain, canary = runs
+    assert np.all(canary["x"][:, ~inside] == np.float32(1234.5))
+    for name, a in canary.items():
+        if name != "x":
+            assert np.all(a[:, ~inside] == 0), name
+        assert np.array_equal(a[:, inside].view(np.uint32), plain[name][:, inside].view(np.uint32)), name
+
+
 @pytest.mark.parametrize("case", ["qhm_beta0_no_grad_term", "omega0", "sgdm_sum_omega1",
                                   "adopt_beta0", "max_replicas"])
 def test_degenerate_hyperparameters(P, case):
