@@ -343,6 +343,7 @@ class MTDAO:
         self.n_padded = lay["n_padded"]
         self.n_states = lay["n_states"]
         self.offsets = lay["offsets"]
+        self.numels = [int(k) for k in numels]
         self.n_mom = int(opt["n_mom"])
 
     def close(self) -> None:
@@ -421,6 +422,24 @@ class MTDAO:
         out = torch.empty((2 * self.M + 2,), dtype=torch.float64, device="cuda")
         mtdao_pseudo_grad_stats(self.h, state, out.data_ptr())
         return out
+
+    def tensor_views(self, flat, shapes):
+        """Views of one flattened [n_padded] vector laid out like this
+        handle's tensor list -- a replica's state (``state_view(s)[m]``) or a
+        row of a gradient buffer -- one per tensor, shaped by ``shapes``
+        (each with the numel given at construction).  The views share the
+        vector's memory: a model can use a replica's parameters in place and
+        write its gradients in place, with no packing copy."""
+        import math
+        if len(shapes) != len(self.numels):
+            raise ValueError("expected %d shapes, got %d" % (len(self.numels), len(shapes)))
+        views = []
+        for off, k, shp in zip(self.offsets, self.numels, shapes):
+            shp = tuple(int(d) for d in shp)
+            if math.prod(shp) != k:
+                raise ValueError("shape %s does not hold %d elements" % (shp, k))
+            views.append(flat[off:off + k].view(shp))
+        return views
 
     def state_ptr(self, state: int, replica: int) -> int:
         return mtdao_get_state_ptr(self.h, state, replica)
