@@ -110,14 +110,16 @@ def test_fused_sync_is_bitwise_equal_to_separate_sync(P, M, gdt):
         b.close()
 
 
+@pytest.mark.parametrize("M", [3, 4, 8])
+@pytest.mark.parametrize("gdt", ["f32", "bf16"])
 @pytest.mark.parametrize("base", ["adam", "sgdm"])
-def test_global_norm_clip_parity(P, base):
+def test_global_norm_clip_parity(P, base, gdt, M):
     # sigma = 1 gives ||g|| ~ 90 >> rho = 1: clipping is active every step
-    w = workload_dict([5000, 3001, 17], 4, base=base, betas=(0.9, 0.999), clip="global_norm",
-                      rho=1.0, px=3, pu=2, pv=3, sigma=1.0)
+    w = workload_dict([5000, 3001, 17], M, base=base, betas=(0.9, 0.999), clip="global_norm",
+                      rho=1.0, px=3, pu=2, pv=3, sigma=1.0, gdt=gdt)
     eng = gpu_run(P, w, 10)
     lay = W.layout(w["shapes"])
-    ref = oracle_run(w["opt"], 4, np.arange(lay["n_padded"]), 10, lay, w, SEED_G, SEED_I)
+    ref = oracle_run(w["opt"], M, np.arange(lay["n_padded"]), 10, lay, w, SEED_G, SEED_I)
     compare(gpu_states(eng, w["opt"]), ref)
     eng.close()
 
@@ -173,12 +175,14 @@ def test_grad_nonfinite_counts(P, gdt):
 
 
 @pytest.mark.parametrize("clip", ["elementwise", "none"])
-def test_adopt_clip_parity(P, clip):
-    w = workload_dict(RAGGED, 4, base="adopt", betas=(0.95, 0.999), beta2=0.9999, clip=clip,
-                      px=6, pu=3, pv=3, lr=2.0 ** -8)
+@pytest.mark.parametrize("gdt", ["f32", "bf16"])
+@pytest.mark.parametrize("M", [2, 4, 8])
+def test_adopt_clip_parity(P, clip, M, gdt):
+    w = workload_dict(RAGGED, M, base="adopt", betas=(0.95, 0.999), beta2=0.9999, clip=clip,
+                      px=6, pu=3, pv=3, lr=2.0 ** -8, gdt=gdt)
     eng = gpu_run(P, w, 20)
     lay = W.layout(w["shapes"])
-    ref = oracle_run(w["opt"], 4, np.arange(lay["n_padded"]), 20, lay, w, SEED_G, SEED_I)
+    ref = oracle_run(w["opt"], M, np.arange(lay["n_padded"]), 20, lay, w, SEED_G, SEED_I)
     compare(gpu_states(eng, w["opt"]), ref)
     eng.close()
 
@@ -197,12 +201,14 @@ def test_adopt_original_ordering_parity(P, clip, M):
     eng.close()
 
 
-def test_alg2_literal_phase_parity(P):
-    w = workload_dict(RAGGED, 4, base="adopt", betas=(0.95,), beta2=0.9999, px=4, pu=3, pv=5,
-                      phase="alg2_literal", lr=2.0 ** -8)
+@pytest.mark.parametrize("M", [3, 4, 8])
+@pytest.mark.parametrize("base", ["adopt", "adam", "sgdm"])
+def test_alg2_literal_phase_parity(P, base, M):
+    w = workload_dict(RAGGED, M, base=base, betas=(0.95, 0.5), beta2=0.9999 if base == "adopt" else 0.999,
+                      px=4, pu=[3, 2], pv=5, phase="alg2_literal", lr=2.0 ** -8)
     eng = gpu_run(P, w, 14)
     lay = W.layout(w["shapes"])
-    ref = oracle_run(w["opt"], 4, np.arange(lay["n_padded"]), 14, lay, w, SEED_G, SEED_I)
+    ref = oracle_run(w["opt"], M, np.arange(lay["n_padded"]), 14, lay, w, SEED_G, SEED_I)
     compare(gpu_states(eng, w["opt"]), ref)
     eng.close()
 
