@@ -415,7 +415,7 @@ def run_ours(args):
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        rate, spent, desc = oracle_sample_rate(w, 1 << 20)
+        rate, spent, desc = oracle_sample_rate(w, 1 << 21)      # ~13 s of one host core
         cpu = {"value": rate, "unit": "params/s", "cores": 1, "kind": "oracle", "sample": desc,
                "seconds": round(spent, 2)}
 
