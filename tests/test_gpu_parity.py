@@ -266,23 +266,27 @@ def test_sync_identity_on_identical_replicas(P, M):
     eng.close()
 
 
+@pytest.mark.parametrize("M,gdt", [(4, "f32"), (8, "bf16"), (3, "bf16")])
 @pytest.mark.parametrize("memory", ["pinned", "pageable"])
-def test_host_gradient_path_is_bitwise_equal(P, memory):
+def test_host_gradient_path_is_bitwise_equal(P, memory, M, gdt):
     """Pinned host gradients are read by the kernel over the host link;
     pageable ones go through the staging copy.  Both equal the device path."""
-    w = workload_dict(RAGGED, 4, betas=(0.9, 0.999), px=3, pu=3, pv=3)
+    w = workload_dict(RAGGED, M, betas=(0.9, 0.999), px=3, pu=3, pv=3, gdt=gdt)
     lay = W.layout(w["shapes"])
     idx = np.arange(lay["n_padded"])
     a = gpu_run(P, w, 7)
-    b = P.MTDAO(w["opt"], 4, w["shapes"])
+    b = P.MTDAO(w["opt"], M, w["shapes"])
     b.set_params(torch.from_numpy(G.init_params(w, lay, SEED_I, idx)).cuda())
+    dt = P.BF16 if gdt == "bf16" else P.F32
     for t in range(7):
         g = np.ascontiguousarray(host_grads(w, lay, SEED_G, t, idx))
+        if gdt == "bf16":
+            g = np.ascontiguousarray(G.to_bf16_bits(g))          # the bf16 bit patterns
         if memory == "pinned":
-            gt = torch.from_numpy(g).pin_memory()
-            b.step_host(gt, 1e-3)
+            gt = torch.from_numpy(g.view(np.int16) if gdt == "bf16" else g).pin_memory()
+            b.step_host(gt.data_ptr(), 1e-3, dtype=dt)
         else:
-            b.step_host(g.ctypes.data, 1e-3, dtype=P.F32)
+            b.step_host(g.ctypes.data, 1e-3, dtype=dt)
         torch.cuda.current_stream().synchronize()
     sa, sb = gpu_states(a, w["opt"]), gpu_states(b, w["opt"])
     for k in sa:
@@ -420,6 +424,61 @@ def test_padding_canaries_are_untouched(P, base, M):
         if name != "x":
             assert np.all(a[:, ~inside] == 0), name
         assert np.array_equal(a[:, inside].view(np.uint32), plain[name][:, inside].view(np.uint32)), name
+
+
+def test_handle_streams_are_respected(P):
+    """A handle created on a side stream, switched to another stream with
+    mtdao_set_stream half-way, and two handles stepping concurrently on two
+    streams all give the bits of the same run on the default stream: every
+    launch and copy goes to the handle's stream."""
+    w = workload_dict(RAGGED, 4, betas=(0.9, 0.99), px=3, pu=[2, 5], pv=4)
+    lay = W.layout(w["shapes"])
+    n = lay["n_padded"]
+    T = 9
+    x0 = torch.from_numpy(G.init_params(w, lay, SEED_I, np.arange(n))).cuda()
+    gs = [to_dev(host_grads(w, lay, SEED_G, t, np.arange(n)), "f32") for t in range(T)]
+    torch.cuda.synchronize()
+
+    def run(eng, stream_for_step):
+        for t in range(T):
+            with torch.cuda.stream(stream_for_step(t)):
+                eng.step(gs[t], 1e-3)
+        return eng
+
+    base = P.MTDAO(w["opt"], 4, w["shapes"])
+    base.set_params(x0)
+    run(base, lambda t: torch.cuda.current_stream())
+    torch.cuda.synchronize()
+    ref = gpu_states(base, w["opt"])
+    base.close()
+
+    s1, s2 = torch.cuda.Stream(), torch.cuda.Stream()
+    eng = P.MTDAO(w["opt"], 4, w["shapes"], stream=s1.cuda_stream)
+    eng.set_params(x0)
+    for t in range(T):
+        if t == 5:
+            s2.wait_stream(s1)
+            P.mtdao_set_stream(eng.h, s2.cuda_stream)
+        P.mtdao_step(eng.h, gs[t].data_ptr(), P.F32, 1e-3, P.mtdao_sync_due(eng.h))
+    s2.synchronize()
+    got = gpu_states(eng, w["opt"])
+    eng.close()
+    for k in ref:
+        assert np.array_equal(got[k].view(np.uint32), ref[k].view(np.uint32)), k
+
+    a = P.MTDAO(w["opt"], 4, w["shapes"], stream=s1.cuda_stream)
+    b = P.MTDAO(w["opt"], 4, w["shapes"], stream=s2.cuda_stream)
+    a.set_params(x0)
+    b.set_params(x0)
+    for t in range(T):                     # interleaved launches, two streams
+        P.mtdao_step(a.h, gs[t].data_ptr(), P.F32, 1e-3, P.mtdao_sync_due(a.h))
+        P.mtdao_step(b.h, gs[t].data_ptr(), P.F32, 1e-3, P.mtdao_sync_due(b.h))
+    torch.cuda.synchronize()
+    for eng in (a, b):
+        got = gpu_states(eng, w["opt"])
+        for k in ref:
+            assert np.array_equal(got[k].view(np.uint32), ref[k].view(np.uint32)), k
+        eng.close()
 
 
 @pytest.mark.parametrize("case", ["qhm_beta0_no_grad_term", "omega0", "sgdm_sum_omega1",
