@@ -296,9 +296,13 @@ int mtdao_sync(mtdao_handle h, uint32_t mask);
  *   [2 + M + m]      <s_m, s_bar>                     (cosine = [2+M+m] /
  *                                                      sqrt([2+m] * [1]))
  * The averaged states are bit-identical to mtdao_sync's.  Sums are
- * fixed-order (bit-reproducible).  Requires M <= 8; with M = 1 the states
- * are left as they are and only the diagnostics are written.  A workspace
- * is allocated on the first call.
+ * fixed-order (bit-reproducible).  With M = 1 the states are left as they
+ * are and only the diagnostics are written.  For M <= 8 the sums are
+ * formed in the averaging pass itself (the sync's traffic, 8 M bytes per
+ * element and state); for larger M each state takes two passes through a
+ * library-owned [n_padded] fp32 scratch that holds the mean (about twice
+ * the traffic), and (s_m - s_bar)^2 is summed as (s_m - s_0)^2 minus
+ * M (s_bar - s_0)^2, in fp64.  Workspaces are allocated on the first call.
  */
 int mtdao_sync_stats(mtdao_handle h, uint32_t mask, double *stats_dev);
 
@@ -327,7 +331,8 @@ int mtdao_track_anchor(mtdao_handle h, uint32_t state_mask);
  * so cos(local, global) = [M+m] / sqrt([m] [2M]) and the relative change of
  * the averaged state over the round = sqrt([2M] / [2M+1]).  Call it before
  * the round's average of that state.  MTDAO_ERR_STATE if the state has no
- * anchor; requires M <= 8.
+ * anchor.  For M > 8 it takes two read-only passes through the scratch of
+ * mtdao_sync_stats.
  */
 int mtdao_pseudo_grad_stats(mtdao_handle h, int32_t state, double *out_dev);
 

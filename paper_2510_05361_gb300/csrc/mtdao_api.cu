@@ -81,6 +81,7 @@ struct mtdao_ctx {
     int norm_blocks = 1;
     double *stats_partial = nullptr;  // diagnostics workspace (allocated on first use)
     size_t stats_cap = 0;
+    float *stats_mean = nullptr;      // M > 8 diagnostics: [n_padded] replica mean (first use)
     float *anchor[2 + MTDAO_MAX_MOM] = {};  // per state: its value at the last average
     // host-gradient staging (mtdao_step_host)
     void *staging[2] = {nullptr, nullptr};
@@ -266,6 +267,7 @@ void release(mtdao_ctx *h) {
     if (h->norm_out) cudaFree(h->norm_out);
     if (h->norm_partial) cudaFree(h->norm_partial);
     if (h->stats_partial) cudaFree(h->stats_partial);
+    if (h->stats_mean) cudaFree(h->stats_mean);
     for (float *a : h->anchor)
         if (a) cudaFree(a);
 }
@@ -508,16 +510,32 @@ static int refresh_anchor(mtdao_ctx *h, uint32_t mask) {
     return MTDAO_OK;
 }
 
+// Diagnostics kernels hold M replicas in registers up to this M; above it
+// they take two passes through a scratch vector.
+constexpr int kStatsRegisterM = 8;
+
 static int ensure_stats_workspace(mtdao_ctx *h) {
-    if (h->stats_partial != nullptr) return MTDAO_OK;
-    const size_t cap = sync_stats_partial_capacity(h->num_sms, h->n_states, h->M);
-    cudaError_t e = cudaMalloc(reinterpret_cast<void **>(&h->stats_partial), cap * sizeof(double));
-    if (e != cudaSuccess) {
-        cudaGetLastError();
-        h->stats_partial = nullptr;
-        return set_error(h, MTDAO_ERR_OOM, "diagnostics workspace: %s", cudaGetErrorString(e));
+    const bool general = h->M > kStatsRegisterM;
+    if (h->stats_partial != nullptr && (!general || h->stats_mean != nullptr)) return MTDAO_OK;
+    if (h->stats_partial == nullptr) {
+        const size_t cap = general ? general_stats_partial_capacity(h->num_sms, h->M)
+                                   : sync_stats_partial_capacity(h->num_sms, h->n_states, h->M);
+        cudaError_t e = cudaMalloc(reinterpret_cast<void **>(&h->stats_partial), cap * sizeof(double));
+        if (e != cudaSuccess) {
+            cudaGetLastError();
+            h->stats_partial = nullptr;
+            return set_error(h, MTDAO_ERR_OOM, "diagnostics workspace: %s", cudaGetErrorString(e));
+        }
+        h->stats_cap = cap;
     }
-    h->stats_cap = cap;
+    if (general) {
+        cudaError_t e = cudaMalloc(reinterpret_cast<void **>(&h->stats_mean), h->n_padded * sizeof(float));
+        if (e != cudaSuccess) {
+            cudaGetLastError();
+            h->stats_mean = nullptr;
+            return set_error(h, MTDAO_ERR_OOM, "diagnostics scratch: %s", cudaGetErrorString(e));
+        }
+    }
     return MTDAO_OK;
 }
 
@@ -670,7 +688,6 @@ extern "C" int mtdao_sync_stats(mtdao_handle h, uint32_t mask, double *stats_dev
     if (stats_dev == nullptr) return set_error(h, MTDAO_ERR_INVALID, "stats is NULL");
     if (mask >> h->n_states) return set_error(h, MTDAO_ERR_INVALID, "sync mask 0x%x has bits beyond "
                                               "the %d states", mask, h->n_states);
-    if (h->M > 8) return set_error(h, MTDAO_ERR_INVALID, "diagnostics support M <= 8 (M = %d)", h->M);
     if (mask == 0) return MTDAO_OK;
     if (int rc = select_device(h)) return rc;
     if (int rc = ensure_stats_workspace(h)) return rc;
@@ -682,7 +699,10 @@ extern "C" int mtdao_sync_stats(mtdao_handle h, uint32_t mask, double *stats_dev
     a.M = h->M;
     for (int s = 0; s < h->n_states; ++s)
         if (mask & (1u << s)) a.sel[a.n_sel++] = s;
-    cudaError_t e = launch_sync_stats(a, h->num_sms, h->stats_partial, h->stats_cap, stats_dev, h->stream);
+    cudaError_t e = h->M > kStatsRegisterM
+                        ? launch_sync_stats_general(a, h->num_sms, h->stats_mean, h->stats_partial, h->stats_cap,
+                                                    stats_dev, h->stream)
+                        : launch_sync_stats(a, h->num_sms, h->stats_partial, h->stats_cap, stats_dev, h->stream);
     if (e != cudaSuccess) return cuda_fail(h, e, "sync with diagnostics launch");
     return refresh_anchor(h, mask);
 }
@@ -725,12 +745,15 @@ extern "C" int mtdao_pseudo_grad_stats(mtdao_handle h, int32_t state, double *ou
     if (state < 0 || state >= h->n_states) return set_error(h, MTDAO_ERR_INVALID, "state %d out of range", state);
     if (h->anchor[state] == nullptr)
         return set_error(h, MTDAO_ERR_STATE, "state %d has no anchor: track it with mtdao_track_anchor", state);
-    if (h->M > 8) return set_error(h, MTDAO_ERR_INVALID, "diagnostics support M <= 8 (M = %d)", h->M);
     if (int rc = select_device(h)) return rc;
     if (int rc = ensure_stats_workspace(h)) return rc;
     const float *x = h->arena + static_cast<int64_t>(state) * h->M * h->n_padded;
-    cudaError_t e = launch_pseudo_grad_stats(x, h->anchor[state], h->n_padded, h->M, h->num_sms,
-                                             h->stats_partial, h->stats_cap, out_dev, h->stream);
+    cudaError_t e = h->M > kStatsRegisterM
+                        ? launch_pseudo_grad_stats_general(x, h->anchor[state], h->n_padded, h->M, h->num_sms,
+                                                           h->stats_mean, h->stats_partial, h->stats_cap,
+                                                           out_dev, h->stream)
+                        : launch_pseudo_grad_stats(x, h->anchor[state], h->n_padded, h->M, h->num_sms,
+                                                   h->stats_partial, h->stats_cap, out_dev, h->stream);
     if (e != cudaSuccess) return cuda_fail(h, e, "change diagnostics launch");
     return MTDAO_OK;
 }

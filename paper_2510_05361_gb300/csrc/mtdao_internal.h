@@ -81,6 +81,18 @@ cudaError_t launch_grad_sqnorm(const void *grads, int grad_dtype, int32_t M, int
                                int blocks_per_replica, double *partial, double *out,
                                float *clip_scale, double rho, cudaStream_t stream);
 
+// Diagnostics for any M (two passes per state through a [n_padded] fp32
+// scratch that holds the replica mean; see reduce_kernels.cu).  Same
+// outputs as launch_sync_stats / launch_pseudo_grad_stats; the averaged
+// states are bit-identical to launch_sync's.  Workspace: partial needs
+// general_stats_partial_capacity() doubles.
+size_t general_stats_partial_capacity(int num_sms, int M);
+cudaError_t launch_sync_stats_general(const SyncArgs &a, int num_sms, float *mean_scratch, double *partial,
+                                      size_t partial_cap, double *stats, cudaStream_t stream);
+cudaError_t launch_pseudo_grad_stats_general(const float *x, const float *anchor, int64_t n, int M, int num_sms,
+                                             float *mean_scratch, double *partial, size_t partial_cap,
+                                             double *stats, cudaStream_t stream);
+
 // Number of NaN / +-Inf gradient values per replica into out[m] (double,
 // exact), with the grid and workspace of launch_grad_sqnorm.
 cudaError_t launch_grad_nonfinite(const void *grads, int grad_dtype, int32_t M, int64_t n_padded,

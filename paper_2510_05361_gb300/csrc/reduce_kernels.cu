@@ -386,6 +386,222 @@ cudaError_t launch_pseudo_grad_stats_t(const float *x, const float *anchor, int6
     return cudaGetLastError();
 }
 
+
+// ---------------------------------------------------------------- diagnostics for any M
+
+// For M above the register-resident kernels' limit the diagnostics take two
+// passes over one state (a [n] fp32 scratch holds the mean between them):
+//   pass 1 (grid-stride over float4 positions): the replica mean of
+//     replica_mean.cuh (the bits mtdao_sync stores), written to the
+//     scratch, and two sums over the elements -- the "global" terms;
+//   pass 2 (grid (blocks, M)): per replica two sums against the scratch
+//     mean -- the "per-replica" terms -- and, for an average, the mean
+//     written over the replica.
+// Each thread accumulates in fp64 (one value per position, added in fixed
+// order), warps and blocks reduce in fixed order, and a finalize kernel
+// adds the block partials in block order: bit-reproducible.
+
+// Deterministic block reduction of two doubles per thread into
+// out[0], out[1] (written by thread 0).
+__device__ void block_sum2(double a, double b, double *out) {
+    __shared__ double part[2][kNormThreads / 32];
+    a = warp_sum(a);
+    b = warp_sum(b);
+    const int w = threadIdx.x >> 5, l = threadIdx.x & 31;
+    if (l == 0) {
+        part[0][w] = a;
+        part[1][w] = b;
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        double ta = 0.0, tb = 0.0;
+        for (int i = 0; i < static_cast<int>(blockDim.x >> 5); ++i) {
+            ta += part[0][i];
+            tb += part[1][i];
+        }
+        out[0] = ta;
+        out[1] = tb;
+    }
+}
+
+// Mean of the M replicas at float4 position e of state s (the runtime-M
+// form of sync_kernel, same operations in the same order); also returns
+// the shifted sum of squares sum_m (s_m - s_0)^2 per element in sq.
+__device__ __forceinline__ float4 mean_and_shifted_sq(const float *s, int64_t n, int M, int64_t e,
+                                                      float4 &s0v, double (&sq)[4]) {
+    float s0[4];
+    to_array(ld_state(s + e), s0);
+    DiffSum pa[4] = {DiffSum(s0[0]), DiffSum(s0[1]), DiffSum(s0[2]), DiffSum(s0[3])};
+    DiffSum pb[4] = {DiffSum(s0[0]), DiffSum(s0[1]), DiffSum(s0[2]), DiffSum(s0[3])};
+#pragma unroll
+    for (int k = 0; k < 4; ++k) sq[k] = 0.0;
+    const int h = M / 2;
+    for (int m = 1; m < M; ++m) {
+        float r[4];
+        to_array(ld_state(s + m * n + e), r);
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+            if (m < h) pa[k].add(r[k]);
+            else pb[k].add(r[k]);
+            const double d = static_cast<double>(r[k]) - static_cast<double>(s0[k]);
+            sq[k] += d * d;
+        }
+    }
+    float mean[4];
+#pragma unroll
+    for (int k = 0; k < 4; ++k)
+        mean[k] = replica_mean_from_parts(s0[k], pa[k].partial(), pb[k].partial(), static_cast<float>(M));
+    s0v = from_array(s0);
+    return from_array(mean);
+}
+
+// Pass 1 of the sync diagnostics: mean -> scratch; per block
+// (sum (s_m - s_bar)^2, sum s_bar^2), the first from the shifted sums:
+// sum_m (s_m - s_bar)^2 = sum_m (s_m - s_0)^2 - M (s_bar - s_0)^2.
+__global__ void __launch_bounds__(kNormThreads) sync_stats_pass1_kernel(const float *s, int64_t n, int M,
+                                                                       float *mean_out, double *partial) {
+    const int64_t nv = n / 4;
+    double q0 = 0.0, q1 = 0.0;
+    for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < nv;
+         i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+        const int64_t e = 4 * i;
+        float4 s0v;
+        double sq[4];
+        const float4 mv = mean_and_shifted_sq(s, n, M, e, s0v, sq);
+        *reinterpret_cast<float4 *>(mean_out + e) = mv;
+        float mean[4], s0[4];
+        to_array(mv, mean);
+        to_array(s0v, s0);
+        double p0 = 0.0, p1 = 0.0;
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+            const double dm = static_cast<double>(mean[k]) - static_cast<double>(s0[k]);
+            p0 += sq[k] - static_cast<double>(M) * dm * dm;
+            p1 += static_cast<double>(mean[k]) * mean[k];
+        }
+        q0 += p0;
+        q1 += p1;
+    }
+    block_sum2(q0, q1, partial + 2 * static_cast<int64_t>(blockIdx.x));
+}
+
+// Pass 2 of the sync diagnostics, replica m = blockIdx.y: per block
+// (sum s_m^2, sum s_m * s_bar); with write_mean the replica is overwritten
+// by the mean (the average itself).
+__global__ void __launch_bounds__(kNormThreads) sync_stats_pass2_kernel(float *s, int64_t n, const float *mean,
+                                                                       int write_mean, double *partial) {
+    const int m = blockIdx.y;
+    const int64_t nv = n / 4;
+    float *rep = s + m * n;
+    double q0 = 0.0, q1 = 0.0;
+    for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < nv;
+         i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+        const int64_t e = 4 * i;
+        const float4 rv = ld_state(rep + e);
+        const float4 mv = *reinterpret_cast<const float4 *>(mean + e);
+        q0 += static_cast<double>(rv.x) * rv.x + static_cast<double>(rv.y) * rv.y +
+              static_cast<double>(rv.z) * rv.z + static_cast<double>(rv.w) * rv.w;
+        q1 += static_cast<double>(rv.x) * mv.x + static_cast<double>(rv.y) * mv.y +
+              static_cast<double>(rv.z) * mv.z + static_cast<double>(rv.w) * mv.w;
+        if (write_mean) st_state(rep + e, mv);
+    }
+    block_sum2(q0, q1, partial + 2 * (static_cast<int64_t>(m) * gridDim.x + blockIdx.x));
+}
+
+// Pass 1 of the change diagnostics: x_bar -> scratch; per block
+// (sum (x_bar - a)^2, sum a^2).
+__global__ void __launch_bounds__(kNormThreads) pseudo_grad_pass1_kernel(const float *x, const float *anchor,
+                                                                        int64_t n, int M, float *mean_out,
+                                                                        double *partial) {
+    const int64_t nv = n / 4;
+    double q0 = 0.0, q1 = 0.0;
+    for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < nv;
+         i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+        const int64_t e = 4 * i;
+        float4 s0v;
+        double sq[4];
+        const float4 mv = mean_and_shifted_sq(x, n, M, e, s0v, sq);
+        *reinterpret_cast<float4 *>(mean_out + e) = mv;
+        const float4 av = __ldcs(reinterpret_cast<const float4 *>(anchor + e));
+        float mean[4], a[4];
+        to_array(mv, mean);
+        to_array(av, a);
+        double p0 = 0.0, p1 = 0.0;
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+            const float glob = mean[k] - a[k];
+            p0 += static_cast<double>(glob) * glob;
+            p1 += static_cast<double>(a[k]) * a[k];
+        }
+        q0 += p0;
+        q1 += p1;
+    }
+    block_sum2(q0, q1, partial + 2 * static_cast<int64_t>(blockIdx.x));
+}
+
+// Pass 2 of the change diagnostics, replica m = blockIdx.y: per block
+// (sum (x_m - a)^2, sum (x_m - a)(x_bar - a)).  Read-only.
+__global__ void __launch_bounds__(kNormThreads) pseudo_grad_pass2_kernel(const float *x, const float *anchor,
+                                                                        int64_t n, const float *mean,
+                                                                        double *partial) {
+    const int m = blockIdx.y;
+    const int64_t nv = n / 4;
+    const float *rep = x + m * n;
+    double q0 = 0.0, q1 = 0.0;
+    for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < nv;
+         i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+        const int64_t e = 4 * i;
+        float r[4], mb[4], a[4];
+        to_array(ld_state(rep + e), r);
+        to_array(*reinterpret_cast<const float4 *>(mean + e), mb);
+        to_array(*reinterpret_cast<const float4 *>(anchor + e), a);
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+            const float loc = r[k] - a[k];
+            const float glob = mb[k] - a[k];
+            q0 += static_cast<double>(loc) * loc;
+            q1 += static_cast<double>(loc) * glob;
+        }
+    }
+    block_sum2(q0, q1, partial + 2 * (static_cast<int64_t>(m) * gridDim.x + blockIdx.x));
+}
+
+// out[g0] = sum_b p1[b][0] (divided by divide_g0 if > 0), out[g1] =
+// sum_b p1[b][1]; out[r0 + m] = sum_b p2[m][b][0], out[r1 + m] =
+// sum_b p2[m][b][1]; block sums added in block order.
+__global__ void general_stats_finalize_kernel(const double *p1, int b1, const double *p2, int b2, int M,
+                                              int g0, int g1, int r0, int r1, int divide_g0, double *out) {
+    if (threadIdx.x == 0) {
+        double t0 = 0.0, t1 = 0.0;
+        for (int b = 0; b < b1; ++b) {
+            t0 += p1[2 * b];
+            t1 += p1[2 * b + 1];
+        }
+        out[g0] = divide_g0 > 0 ? t0 / divide_g0 : t0;
+        out[g1] = t1;
+    }
+    for (int m = threadIdx.x; m < M; m += blockDim.x) {
+        double t0 = 0.0, t1 = 0.0;
+        for (int b = 0; b < b2; ++b) {
+            t0 += p2[2 * (static_cast<int64_t>(m) * b2 + b)];
+            t1 += p2[2 * (static_cast<int64_t>(m) * b2 + b) + 1];
+        }
+        out[r0 + m] = t0;
+        out[r1 + m] = t1;
+    }
+}
+
+struct GeneralGrid {
+    int b1, b2;
+};
+
+GeneralGrid general_grid(int num_sms, int M, int64_t n) {
+    const int64_t need = (n / 4 + kNormThreads - 1) / kNormThreads;
+    int64_t b1 = 4 * static_cast<int64_t>(num_sms), b2 = b1 / M;
+    if (b1 > need) b1 = need;
+    if (b2 > need) b2 = need;
+    return {static_cast<int>(b1 < 1 ? 1 : b1), static_cast<int>(b2 < 1 ? 1 : b2)};
+}
 }  // namespace
 
 cudaError_t launch_pseudo_grad_stats(const float *x, const float *anchor, int64_t n, int M, int num_sms,
@@ -465,6 +681,47 @@ cudaError_t launch_grad_sqnorm(const void *grads, int grad_dtype, int32_t M, int
     if (e != cudaSuccess) return e;
     sqnorm_finalize_kernel<<<M, kNormThreads, 0, stream>>>(partial, blocks_per_replica, out, clip_scale,
                                                           rho);
+    return cudaGetLastError();
+}
+
+
+size_t general_stats_partial_capacity(int num_sms, int M) {
+    return static_cast<size_t>(2) * (4 * static_cast<size_t>(num_sms) + static_cast<size_t>(M) *
+                                     (4 * static_cast<size_t>(num_sms) / (M > 0 ? M : 1) + 1));
+}
+
+cudaError_t launch_sync_stats_general(const SyncArgs &a, int num_sms, float *mean_scratch, double *partial,
+                                      size_t partial_cap, double *stats, cudaStream_t stream) {
+    const int M = a.M;
+    const int Q = 2 + 2 * M;
+    const GeneralGrid g = general_grid(num_sms, M, a.n_padded);
+    if (static_cast<size_t>(2) * (g.b1 + static_cast<size_t>(g.b2) * M) > partial_cap)
+        return cudaErrorInvalidValue;
+    double *p1 = partial, *p2 = partial + 2 * g.b1;
+    for (int k = 0; k < a.n_sel; ++k) {
+        float *s = a.arena + static_cast<int64_t>(a.sel[k]) * a.stride;
+        sync_stats_pass1_kernel<<<g.b1, kNormThreads, 0, stream>>>(s, a.n_padded, M, mean_scratch, p1);
+        sync_stats_pass2_kernel<<<dim3(g.b2, M), kNormThreads, 0, stream>>>(s, a.n_padded, mean_scratch,
+                                                                            M > 1 ? 1 : 0, p2);
+        general_stats_finalize_kernel<<<1, 256, 0, stream>>>(p1, g.b1, p2, g.b2, M, 0, 1, 2, 2 + M, M,
+                                                             stats + static_cast<int64_t>(k) * Q);
+        cudaError_t e = cudaGetLastError();
+        if (e != cudaSuccess) return e;
+    }
+    return cudaSuccess;
+}
+
+cudaError_t launch_pseudo_grad_stats_general(const float *x, const float *anchor, int64_t n, int M, int num_sms,
+                                             float *mean_scratch, double *partial, size_t partial_cap,
+                                             double *stats, cudaStream_t stream) {
+    const GeneralGrid g = general_grid(num_sms, M, n);
+    if (static_cast<size_t>(2) * (g.b1 + static_cast<size_t>(g.b2) * M) > partial_cap)
+        return cudaErrorInvalidValue;
+    double *p1 = partial, *p2 = partial + 2 * g.b1;
+    pseudo_grad_pass1_kernel<<<g.b1, kNormThreads, 0, stream>>>(x, anchor, n, M, mean_scratch, p1);
+    pseudo_grad_pass2_kernel<<<dim3(g.b2, M), kNormThreads, 0, stream>>>(x, anchor, n, mean_scratch, p2);
+    general_stats_finalize_kernel<<<1, 256, 0, stream>>>(p1, g.b1, p2, g.b2, M, 2 * M, 2 * M + 1, 0, M, 0,
+                                                         stats);
     return cudaGetLastError();
 }
 

@@ -33,9 +33,12 @@ def _fill(eng, rng, spread):
     return vals
 
 
-@pytest.mark.parametrize("M", [1, 2, 3, 4, 8])
+@pytest.mark.parametrize("M", [1, 2, 3, 4, 8, 9, 16, 37, 256])
 def test_sync_stats_match_oracle_and_plain_sync(P, M):
-    shapes = [70001, 999, 4096]
+    """M <= 8: one pass with the replicas in registers; M > 8: two passes
+    through a scratch mean.  Both match the oracle's definitions and leave
+    the states bit-identical to the plain average."""
+    shapes = [70001, 999, 4096] if M <= 37 else [7001, 99, 1024]
     w = workload_dict(shapes, M, betas=(0.9, 0.99))
     a = P.MTDAO(w["opt"], M, shapes)
     b = P.MTDAO(w["opt"], M, shapes)
@@ -92,14 +95,8 @@ def test_sync_stats_cosine_and_variance_during_training(P):
     eng.close()
 
 
-def test_sync_stats_rejects_large_M_and_bad_masks(P):
-    w = workload_dict([1024], 9, betas=(0.9,))
-    eng = P.MTDAO(w["opt"], 9, w["shapes"])
+def test_sync_stats_rejects_bad_masks(P):
     out = torch.zeros(64, dtype=torch.float64, device="cuda")
-    with pytest.raises(P.MTDAOError) as e:
-        P.mtdao_sync_stats(eng.h, 1, out.data_ptr())
-    assert e.value.code == P.ERR_INVALID
-    eng.close()
     w = workload_dict([1024], 2, betas=(0.9,))
     eng = P.MTDAO(w["opt"], 2, w["shapes"])
     with pytest.raises(P.MTDAOError):
@@ -107,7 +104,7 @@ def test_sync_stats_rejects_large_M_and_bad_masks(P):
     eng.close()
 
 
-@pytest.mark.parametrize("M", [2, 4, 8])
+@pytest.mark.parametrize("M", [2, 4, 8, 9, 16])
 def test_pseudo_grad_stats_against_oracle(P, M):
     """Anchor = parameters at the last average; mid-round diagnostics of the
     pseudo-gradients match the oracle's definitions on the same values."""
