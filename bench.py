@@ -370,18 +370,14 @@ def run_ours(args):
     sync_gbs = sync_bytes / (statistics.median(sync_ms) / 1e3) / 1e9
 
     # the same average with the cross-worker diagnostics formed in its pass
-    stats_ms = []
-    if M <= 8:
-        stats_out = torch.empty((n_states, 2 + 2 * M), dtype=torch.float64, device="cuda")
-        stats_ms = launches(lambda: P.mtdao_sync_stats(eng.h, all_mask, stats_out.data_ptr()))
+    stats_out = torch.empty((n_states, 2 + 2 * M), dtype=torch.float64, device="cuda")
+    stats_ms = launches(lambda: P.mtdao_sync_stats(eng.h, all_mask, stats_out.data_ptr()))
 
     # pseudo-gradient diagnostics: a read-only pass over x and the anchor
-    pg_ms = []
-    if M <= 8:
-        P.mtdao_track_anchor(eng.h, 1)
-        pg_out = torch.empty((2 * M + 2,), dtype=torch.float64, device="cuda")
-        pg_ms = launches(lambda: P.mtdao_pseudo_grad_stats(eng.h, 0, pg_out.data_ptr()))
-        P.mtdao_track_anchor(eng.h, 0)
+    P.mtdao_track_anchor(eng.h, 1)
+    pg_out = torch.empty((2 * M + 2,), dtype=torch.float64, device="cuda")
+    pg_ms = launches(lambda: P.mtdao_pseudo_grad_stats(eng.h, 0, pg_out.data_ptr()))
+    P.mtdao_track_anchor(eng.h, 0)
     pg_bytes = (M + 1) * n * 4
 
     # S0: per-replica gradient sum of squares (the clip(g, rho) pre-pass) and

@@ -393,201 +393,239 @@ cudaError_t launch_pseudo_grad_stats_t(const float *x, const float *anchor, int6
 // passes over one state (a [n] fp32 scratch holds the mean between them):
 //   pass 1 (grid-stride over float4 positions): the replica mean of
 //     replica_mean.cuh (the bits mtdao_sync stores), written to the
-//     scratch, and two sums over the elements -- the "global" terms;
-//   pass 2 (grid (blocks, M)): per replica two sums against the scratch
-//     mean -- the "per-replica" terms -- and, for an average, the mean
-//     written over the replica.
-// Each thread accumulates in fp64 (one value per position, added in fixed
-// order), warps and blocks reduce in fixed order, and a finalize kernel
-// adds the block partials in block order: bit-reproducible.
+//     scratch, and the sums that need only the mean (and the anchor);
+//   pass 2 (grid (blocks, M)): per replica the sums against the scratch
+//     mean and, for an average, the mean written over the replica.
+// As in the one-pass kernels, each position's four elements are summed in
+// fp32, each thread accumulates its positions with Kahan compensation, and
+// warps, blocks and a finalize kernel reduce in fp64 in fixed order:
+// bit-reproducible.  (GB300's fp64 rate is far below its fp32 rate, so the
+// per-element work stays in fp32.)
 
-// Deterministic block reduction of two doubles per thread into
-// out[0], out[1] (written by thread 0).
-__device__ void block_sum2(double a, double b, double *out) {
-    __shared__ double part[2][kNormThreads / 32];
-    a = warp_sum(a);
-    b = warp_sum(b);
+// Deterministic block reduction of K doubles per thread into out[0..K)
+// (written by thread 0).
+template <int K>
+__device__ void block_sum_k(const double (&v)[K], double *out) {
+    __shared__ double part[K][kNormThreads / 32];
     const int w = threadIdx.x >> 5, l = threadIdx.x & 31;
-    if (l == 0) {
-        part[0][w] = a;
-        part[1][w] = b;
+#pragma unroll
+    for (int k = 0; k < K; ++k) {
+        const double x = warp_sum(v[k]);
+        if (l == 0) part[k][w] = x;
     }
     __syncthreads();
     if (threadIdx.x == 0) {
-        double ta = 0.0, tb = 0.0;
-        for (int i = 0; i < static_cast<int>(blockDim.x >> 5); ++i) {
-            ta += part[0][i];
-            tb += part[1][i];
+#pragma unroll
+        for (int k = 0; k < K; ++k) {
+            double t = 0.0;
+            for (int i = 0; i < static_cast<int>(blockDim.x >> 5); ++i) t += part[k][i];
+            out[k] = t;
         }
-        out[0] = ta;
-        out[1] = tb;
     }
 }
 
-// Mean of the M replicas at float4 position e of state s (the runtime-M
-// form of sync_kernel, same operations in the same order); also returns
-// the shifted sum of squares sum_m (s_m - s_0)^2 per element in sq.
-__device__ __forceinline__ float4 mean_and_shifted_sq(const float *s, int64_t n, int M, int64_t e,
-                                                      float4 &s0v, double (&sq)[4]) {
+// Mean of the M replicas at float4 position e of state s: the runtime-M
+// form of sync_kernel, the same operations in the same order.
+__device__ __forceinline__ float4 replica_mean4(const float *s, int64_t n, int M, int64_t e) {
     float s0[4];
     to_array(ld_state(s + e), s0);
     DiffSum pa[4] = {DiffSum(s0[0]), DiffSum(s0[1]), DiffSum(s0[2]), DiffSum(s0[3])};
     DiffSum pb[4] = {DiffSum(s0[0]), DiffSum(s0[1]), DiffSum(s0[2]), DiffSum(s0[3])};
-#pragma unroll
-    for (int k = 0; k < 4; ++k) sq[k] = 0.0;
     const int h = M / 2;
-    for (int m = 1; m < M; ++m) {
-        float r[4];
-        to_array(ld_state(s + m * n + e), r);
+    for (int m = 1; m < M; m += 4) {          // four replicas' loads in flight, added in order
+        float r[4][4];
 #pragma unroll
-        for (int k = 0; k < 4; ++k) {
-            if (m < h) pa[k].add(r[k]);
-            else pb[k].add(r[k]);
-            const double d = static_cast<double>(r[k]) - static_cast<double>(s0[k]);
-            sq[k] += d * d;
+        for (int u = 0; u < 4; ++u)
+            if (m + u < M) to_array(ld_state(s + (m + u) * n + e), r[u]);
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            if (m + u >= M) break;
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+                if (m + u < h) pa[k].add(r[u][k]);
+                else pb[k].add(r[u][k]);
+            }
         }
     }
     float mean[4];
 #pragma unroll
     for (int k = 0; k < 4; ++k)
         mean[k] = replica_mean_from_parts(s0[k], pa[k].partial(), pb[k].partial(), static_cast<float>(M));
-    s0v = from_array(s0);
     return from_array(mean);
 }
 
-// Pass 1 of the sync diagnostics: mean -> scratch; per block
-// (sum (s_m - s_bar)^2, sum s_bar^2), the first from the shifted sums:
-// sum_m (s_m - s_bar)^2 = sum_m (s_m - s_0)^2 - M (s_bar - s_0)^2.
-__global__ void __launch_bounds__(kNormThreads) sync_stats_pass1_kernel(const float *s, int64_t n, int M,
+// Positions a pass-2 thread loads before it accumulates them (i, i + T,
+// i + 2T, ...: the order of a plain grid-stride loop): four for the sync
+// diagnostics (two float4 loads per position), two for the change
+// diagnostics (three per position, within 64 registers).
+constexpr int kPass2Unroll = 4;
+constexpr int kPass2UnrollChange = 2;
+
+// Pass 1 of the sync diagnostics: mean -> scratch; per block sum s_bar^2.
+__global__ void __launch_bounds__(kNormThreads, 4) sync_stats_pass1_kernel(const float *s, int64_t n, int M,
                                                                        float *mean_out, double *partial) {
     const int64_t nv = n / 4;
-    double q0 = 0.0, q1 = 0.0;
+    Kahan q;
     for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < nv;
          i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
         const int64_t e = 4 * i;
-        float4 s0v;
-        double sq[4];
-        const float4 mv = mean_and_shifted_sq(s, n, M, e, s0v, sq);
+        const float4 mv = replica_mean4(s, n, M, e);
         *reinterpret_cast<float4 *>(mean_out + e) = mv;
-        float mean[4], s0[4];
-        to_array(mv, mean);
-        to_array(s0v, s0);
-        double p0 = 0.0, p1 = 0.0;
-#pragma unroll
-        for (int k = 0; k < 4; ++k) {
-            const double dm = static_cast<double>(mean[k]) - static_cast<double>(s0[k]);
-            p0 += sq[k] - static_cast<double>(M) * dm * dm;
-            p1 += static_cast<double>(mean[k]) * mean[k];
-        }
-        q0 += p0;
-        q1 += p1;
+        q.add(fmaf(mv.x, mv.x, fmaf(mv.y, mv.y, fmaf(mv.z, mv.z, __fmul_rn(mv.w, mv.w)))));
     }
-    block_sum2(q0, q1, partial + 2 * static_cast<int64_t>(blockIdx.x));
+    const double v[1] = {q.value()};
+    block_sum_k<1>(v, partial + blockIdx.x);
 }
 
 // Pass 2 of the sync diagnostics, replica m = blockIdx.y: per block
-// (sum s_m^2, sum s_m * s_bar); with write_mean the replica is overwritten
-// by the mean (the average itself).
-__global__ void __launch_bounds__(kNormThreads) sync_stats_pass2_kernel(float *s, int64_t n, const float *mean,
+// (sum (s_m - s_bar)^2, sum s_m^2, sum s_m * s_bar); with write_mean the
+// replica is overwritten by the mean (the average itself).
+__global__ void __launch_bounds__(kNormThreads, 4) sync_stats_pass2_kernel(float *s, int64_t n, const float *mean,
                                                                        int write_mean, double *partial) {
     const int m = blockIdx.y;
     const int64_t nv = n / 4;
+    const int64_t T = static_cast<int64_t>(gridDim.x) * blockDim.x;
     float *rep = s + m * n;
-    double q0 = 0.0, q1 = 0.0;
-    for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < nv;
-         i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
-        const int64_t e = 4 * i;
-        const float4 rv = ld_state(rep + e);
-        const float4 mv = *reinterpret_cast<const float4 *>(mean + e);
-        q0 += static_cast<double>(rv.x) * rv.x + static_cast<double>(rv.y) * rv.y +
-              static_cast<double>(rv.z) * rv.z + static_cast<double>(rv.w) * rv.w;
-        q1 += static_cast<double>(rv.x) * mv.x + static_cast<double>(rv.y) * mv.y +
-              static_cast<double>(rv.z) * mv.z + static_cast<double>(rv.w) * mv.w;
-        if (write_mean) st_state(rep + e, mv);
+    Kahan q0, q1, q2;
+    for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < nv; i += kPass2Unroll * T) {
+        float4 rv[kPass2Unroll], mv[kPass2Unroll];
+#pragma unroll
+        for (int u = 0; u < kPass2Unroll; ++u)
+            if (i + u * T < nv) {
+                rv[u] = ld_state(rep + 4 * (i + u * T));
+                mv[u] = *reinterpret_cast<const float4 *>(mean + 4 * (i + u * T));
+            }
+#pragma unroll
+        for (int u = 0; u < kPass2Unroll; ++u) {
+            if (i + u * T >= nv) break;
+            float r[4], mb[4];
+            to_array(rv[u], r);
+            to_array(mv[u], mb);
+            float p0 = 0.0f, p1 = 0.0f, p2 = 0.0f;
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+                const float dv = r[k] - mb[k];
+                p0 = fmaf(dv, dv, p0);
+                p1 = fmaf(r[k], r[k], p1);
+                p2 = fmaf(r[k], mb[k], p2);
+            }
+            q0.add(p0);
+            q1.add(p1);
+            q2.add(p2);
+            if (write_mean) st_state(rep + 4 * (i + u * T), mv[u]);
+        }
     }
-    block_sum2(q0, q1, partial + 2 * (static_cast<int64_t>(m) * gridDim.x + blockIdx.x));
+    const double v[3] = {q0.value(), q1.value(), q2.value()};
+    block_sum_k<3>(v, partial + 3 * (static_cast<int64_t>(m) * gridDim.x + blockIdx.x));
 }
 
 // Pass 1 of the change diagnostics: x_bar -> scratch; per block
 // (sum (x_bar - a)^2, sum a^2).
-__global__ void __launch_bounds__(kNormThreads) pseudo_grad_pass1_kernel(const float *x, const float *anchor,
+__global__ void __launch_bounds__(kNormThreads, 4) pseudo_grad_pass1_kernel(const float *x, const float *anchor,
                                                                         int64_t n, int M, float *mean_out,
                                                                         double *partial) {
     const int64_t nv = n / 4;
-    double q0 = 0.0, q1 = 0.0;
+    Kahan q0, q1;
     for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < nv;
          i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
         const int64_t e = 4 * i;
-        float4 s0v;
-        double sq[4];
-        const float4 mv = mean_and_shifted_sq(x, n, M, e, s0v, sq);
+        const float4 mv = replica_mean4(x, n, M, e);
         *reinterpret_cast<float4 *>(mean_out + e) = mv;
-        const float4 av = __ldcs(reinterpret_cast<const float4 *>(anchor + e));
         float mean[4], a[4];
         to_array(mv, mean);
-        to_array(av, a);
-        double p0 = 0.0, p1 = 0.0;
+        to_array(__ldcs(reinterpret_cast<const float4 *>(anchor + e)), a);
+        float p0 = 0.0f, p1 = 0.0f;
 #pragma unroll
         for (int k = 0; k < 4; ++k) {
             const float glob = mean[k] - a[k];
-            p0 += static_cast<double>(glob) * glob;
-            p1 += static_cast<double>(a[k]) * a[k];
+            p0 = fmaf(glob, glob, p0);
+            p1 = fmaf(a[k], a[k], p1);
         }
-        q0 += p0;
-        q1 += p1;
+        q0.add(p0);
+        q1.add(p1);
     }
-    block_sum2(q0, q1, partial + 2 * static_cast<int64_t>(blockIdx.x));
+    const double v[2] = {q0.value(), q1.value()};
+    block_sum_k<2>(v, partial + 2 * static_cast<int64_t>(blockIdx.x));
 }
 
 // Pass 2 of the change diagnostics, replica m = blockIdx.y: per block
 // (sum (x_m - a)^2, sum (x_m - a)(x_bar - a)).  Read-only.
-__global__ void __launch_bounds__(kNormThreads) pseudo_grad_pass2_kernel(const float *x, const float *anchor,
+__global__ void __launch_bounds__(kNormThreads, 4) pseudo_grad_pass2_kernel(const float *x, const float *anchor,
                                                                         int64_t n, const float *mean,
                                                                         double *partial) {
     const int m = blockIdx.y;
     const int64_t nv = n / 4;
+    const int64_t T = static_cast<int64_t>(gridDim.x) * blockDim.x;
     const float *rep = x + m * n;
-    double q0 = 0.0, q1 = 0.0;
-    for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < nv;
-         i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
-        const int64_t e = 4 * i;
-        float r[4], mb[4], a[4];
-        to_array(ld_state(rep + e), r);
-        to_array(*reinterpret_cast<const float4 *>(mean + e), mb);
-        to_array(*reinterpret_cast<const float4 *>(anchor + e), a);
+    Kahan q0, q1;
+    for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < nv; i += kPass2UnrollChange * T) {
+        float4 rv[kPass2UnrollChange], mv[kPass2UnrollChange], av[kPass2UnrollChange];
 #pragma unroll
-        for (int k = 0; k < 4; ++k) {
-            const float loc = r[k] - a[k];
-            const float glob = mb[k] - a[k];
-            q0 += static_cast<double>(loc) * loc;
-            q1 += static_cast<double>(loc) * glob;
+        for (int u = 0; u < kPass2UnrollChange; ++u)
+            if (i + u * T < nv) {
+                const int64_t e = 4 * (i + u * T);
+                rv[u] = ld_state(rep + e);
+                mv[u] = *reinterpret_cast<const float4 *>(mean + e);
+                av[u] = *reinterpret_cast<const float4 *>(anchor + e);
+            }
+#pragma unroll
+        for (int u = 0; u < kPass2UnrollChange; ++u) {
+            if (i + u * T >= nv) break;
+            float r[4], mb[4], a[4];
+            to_array(rv[u], r);
+            to_array(mv[u], mb);
+            to_array(av[u], a);
+            float p0 = 0.0f, p1 = 0.0f;
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+                const float loc = r[k] - a[k];
+                const float glob = mb[k] - a[k];
+                p0 = fmaf(loc, loc, p0);
+                p1 = fmaf(loc, glob, p1);
+            }
+            q0.add(p0);
+            q1.add(p1);
         }
     }
-    block_sum2(q0, q1, partial + 2 * (static_cast<int64_t>(m) * gridDim.x + blockIdx.x));
+    const double v[2] = {q0.value(), q1.value()};
+    block_sum_k<2>(v, partial + 2 * (static_cast<int64_t>(m) * gridDim.x + blockIdx.x));
 }
 
-// out[g0] = sum_b p1[b][0] (divided by divide_g0 if > 0), out[g1] =
-// sum_b p1[b][1]; out[r0 + m] = sum_b p2[m][b][0], out[r1 + m] =
-// sum_b p2[m][b][1]; block sums added in block order.
+// Adds block partials in block order.  p1 holds K1 values per pass-1
+// block, p2 K2 values per (replica, pass-2 block).  For t < K1:
+// out[g[t]] = sum_b p1[b][t]; for t < K2 and each replica m:
+// out[r[t] + m] = sum_b p2[m][b][t], except that t_sum (if >= 0) is
+// summed over the replicas too and divided by M into out[sum_to]
+// instead.
+struct FinalizeMap {
+    int K1, K2;
+    int g[2];
+    int r[3];
+    int t_sum, sum_to;
+};
+
 __global__ void general_stats_finalize_kernel(const double *p1, int b1, const double *p2, int b2, int M,
-                                              int g0, int g1, int r0, int r1, int divide_g0, double *out) {
+                                              FinalizeMap f, double *out) {
     if (threadIdx.x == 0) {
-        double t0 = 0.0, t1 = 0.0;
-        for (int b = 0; b < b1; ++b) {
-            t0 += p1[2 * b];
-            t1 += p1[2 * b + 1];
+        for (int t = 0; t < f.K1; ++t) {
+            double acc = 0.0;
+            for (int b = 0; b < b1; ++b) acc += p1[b * f.K1 + t];
+            out[f.g[t]] = acc;
         }
-        out[g0] = divide_g0 > 0 ? t0 / divide_g0 : t0;
-        out[g1] = t1;
+        if (f.t_sum >= 0) {
+            double acc = 0.0;
+            for (int m = 0; m < M; ++m)
+                for (int b = 0; b < b2; ++b) acc += p2[(static_cast<int64_t>(m) * b2 + b) * f.K2 + f.t_sum];
+            out[f.sum_to] = acc / M;
+        }
     }
     for (int m = threadIdx.x; m < M; m += blockDim.x) {
-        double t0 = 0.0, t1 = 0.0;
-        for (int b = 0; b < b2; ++b) {
-            t0 += p2[2 * (static_cast<int64_t>(m) * b2 + b)];
-            t1 += p2[2 * (static_cast<int64_t>(m) * b2 + b) + 1];
+        for (int t = 0; t < f.K2; ++t) {
+            if (t == f.t_sum) continue;
+            double acc = 0.0;
+            for (int b = 0; b < b2; ++b) acc += p2[(static_cast<int64_t>(m) * b2 + b) * f.K2 + t];
+            out[f.r[t] + m] = acc;
         }
-        out[r0 + m] = t0;
-        out[r1 + m] = t1;
     }
 }
 
@@ -686,8 +724,9 @@ cudaError_t launch_grad_sqnorm(const void *grads, int grad_dtype, int32_t M, int
 
 
 size_t general_stats_partial_capacity(int num_sms, int M) {
-    return static_cast<size_t>(2) * (4 * static_cast<size_t>(num_sms) + static_cast<size_t>(M) *
-                                     (4 * static_cast<size_t>(num_sms) / (M > 0 ? M : 1) + 1));
+    const size_t b1 = 4 * static_cast<size_t>(num_sms);
+    const size_t b2 = b1 / static_cast<size_t>(M > 0 ? M : 1) + 1;
+    return 2 * b1 + 3 * b2 * static_cast<size_t>(M);
 }
 
 cudaError_t launch_sync_stats_general(const SyncArgs &a, int num_sms, float *mean_scratch, double *partial,
@@ -695,15 +734,16 @@ cudaError_t launch_sync_stats_general(const SyncArgs &a, int num_sms, float *mea
     const int M = a.M;
     const int Q = 2 + 2 * M;
     const GeneralGrid g = general_grid(num_sms, M, a.n_padded);
-    if (static_cast<size_t>(2) * (g.b1 + static_cast<size_t>(g.b2) * M) > partial_cap)
-        return cudaErrorInvalidValue;
-    double *p1 = partial, *p2 = partial + 2 * g.b1;
+    if (static_cast<size_t>(g.b1) + 3 * static_cast<size_t>(g.b2) * M > partial_cap) return cudaErrorInvalidValue;
+    double *p1 = partial, *p2 = partial + g.b1;
+    // stats row: [0] variance (sum over replicas / M), [1] s_bar^2, [2 + m] s_m^2, [2 + M + m] s_m s_bar
+    FinalizeMap f = {1, 3, {1, 0}, {0, 2, 2 + M}, 0, 0};
     for (int k = 0; k < a.n_sel; ++k) {
         float *s = a.arena + static_cast<int64_t>(a.sel[k]) * a.stride;
         sync_stats_pass1_kernel<<<g.b1, kNormThreads, 0, stream>>>(s, a.n_padded, M, mean_scratch, p1);
         sync_stats_pass2_kernel<<<dim3(g.b2, M), kNormThreads, 0, stream>>>(s, a.n_padded, mean_scratch,
                                                                             M > 1 ? 1 : 0, p2);
-        general_stats_finalize_kernel<<<1, 256, 0, stream>>>(p1, g.b1, p2, g.b2, M, 0, 1, 2, 2 + M, M,
+        general_stats_finalize_kernel<<<1, 256, 0, stream>>>(p1, g.b1, p2, g.b2, M, f,
                                                              stats + static_cast<int64_t>(k) * Q);
         cudaError_t e = cudaGetLastError();
         if (e != cudaSuccess) return e;
@@ -715,13 +755,14 @@ cudaError_t launch_pseudo_grad_stats_general(const float *x, const float *anchor
                                              float *mean_scratch, double *partial, size_t partial_cap,
                                              double *stats, cudaStream_t stream) {
     const GeneralGrid g = general_grid(num_sms, M, n);
-    if (static_cast<size_t>(2) * (g.b1 + static_cast<size_t>(g.b2) * M) > partial_cap)
+    if (2 * static_cast<size_t>(g.b1) + 2 * static_cast<size_t>(g.b2) * M > partial_cap)
         return cudaErrorInvalidValue;
     double *p1 = partial, *p2 = partial + 2 * g.b1;
+    // out: [m] (x_m - a)^2, [M + m] (x_m - a)(x_bar - a), [2M] (x_bar - a)^2, [2M + 1] a^2
+    FinalizeMap f = {2, 2, {2 * M, 2 * M + 1}, {0, M, 0}, -1, 0};
     pseudo_grad_pass1_kernel<<<g.b1, kNormThreads, 0, stream>>>(x, anchor, n, M, mean_scratch, p1);
     pseudo_grad_pass2_kernel<<<dim3(g.b2, M), kNormThreads, 0, stream>>>(x, anchor, n, mean_scratch, p2);
-    general_stats_finalize_kernel<<<1, 256, 0, stream>>>(p1, g.b1, p2, g.b2, M, 2 * M, 2 * M + 1, 0, M, 0,
-                                                         stats);
+    general_stats_finalize_kernel<<<1, 256, 0, stream>>>(p1, g.b1, p2, g.b2, M, f, stats);
     return cudaGetLastError();
 }
 
