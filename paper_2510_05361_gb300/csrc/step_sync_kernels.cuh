@@ -1,11 +1,11 @@
 // step_sync_kernels.cuh -- the local step with the replica average fused in.
 //
-// step_sync_kernel is element-major: a lane updates the same few elements of
-// all M replicas (M <= 4) or, for M = 8, of 4 replicas while the lane 16
-// places away holds the other 4 (see FusedShape), with the update of
-// step_kernels.cuh; then it writes each state due for averaging as the
-// replica mean (E_m[.] of Algorithms 1-3) instead of the local values.  The
-// average costs no HBM traffic beyond the step's own.
+// step_sync_kernel is element-major: a lane updates the same few elements
+// of all M replicas (M = 2, 3, 4) or, for M = 6 and 8, of half of them
+// while the lane 16 places away holds the other half (see FusedShape), with
+// the update of step_kernels.cuh; then it writes each state due for
+// averaging as the replica mean (E_m[.] of Algorithms 1-3) instead of the
+// local values.  The average costs no HBM traffic beyond the step's own.
 #pragma once
 
 #include "replica_mean.cuh"
@@ -15,12 +15,17 @@ namespace mtdao {
 
 // ---------------------------------------------------------------- fused step + sync
 
-// Layout of the fused kernel's work.  A lane holds V = 4 consecutive
-// elements (128-bit accesses) of R replicas:
-//   M = 2, 4 : one lane group, R = M;
-//   M = 8    : two lane groups (half-warps), R = 4: lanes q and q + 16 hold
-//              the same elements, replicas 0..3 and 4..7, and combine their
-//              parts of the average by shuffles.
+// Layout of the fused kernel's work.  A lane holds V consecutive elements
+// of R replicas:
+//   M = 2, 3, 4 : one lane group, R = M, V = 4 (128-bit accesses);
+//   M = 6, 8    : two lane groups (half-warps), R = M / 2: lanes q and
+//                 q + 16 hold the same elements, replicas 0..R-1 and R..M-1
+//                 -- exactly the two parts of the compensated mean of
+//                 replica_mean.cuh -- and combine them by shuffles; V = 4
+//                 for M = 8, V = 2 for M = 6 (three replicas of four
+//                 elements spilled registers).
+// M = 5 and 7 (one lane group of 5 or 7 replicas spills even at V = 2) and
+// M > 8 take the plain step followed by the standalone average.
 // The states are visited one after another (state_order); the next
 // state's loads are issued before the current state is updated and stored,
 // so two states' loads are in flight per lane within the 128-register cap.
@@ -31,20 +36,54 @@ namespace mtdao {
 // the same with or without it.
 template <int M>
 struct FusedShape {
-    static constexpr int G = M == 8 ? 2 : 1;      // lane groups per warp
-    static constexpr int R = M / G;               // replicas per lane
-    static constexpr int V = 4;                   // elements per lane
-    static constexpr int kLanes = 32 / G;         // lanes per group
-    static constexpr int kChunk = kLanes * V;     // elements per warp iteration
+    static_assert(M == 2 || M == 3 || M == 4 || M == 6 || M == 8, "no fused shape for this M");
+    static constexpr int G = (M == 6 || M == 8) ? 2 : 1;   // lane groups per warp
+    static constexpr int R = M / G;                         // replicas per lane
+    static constexpr int V = M == 6 ? 2 : 4;                // elements per lane
+    static constexpr int kLanes = 32 / G;                   // lanes per group
+    static constexpr int kChunk = kLanes * V;               // elements per warp iteration
 };
 
-__device__ __forceinline__ void ld_v(const float *p, float *a) { to_array(ld_state(p), a); }
-__device__ __forceinline__ void st_v(float *p, const float *a) { st_state(p, from_array(a)); }
+template <int V>
+__device__ __forceinline__ void ld_v(const float *p, float *a) {
+    if constexpr (V == 4) {
+        to_array(ld_state(p), a);
+    } else {
+        const float2 t = __ldcs(reinterpret_cast<const float2 *>(p));
+        a[0] = t.x;
+        a[1] = t.y;
+    }
+}
+template <int V>
+__device__ __forceinline__ void st_v(float *p, const float *a) {
+    if constexpr (V == 4)
+        st_state(p, from_array(a));
+    else
+        __stcs(reinterpret_cast<float2 *>(p), make_float2(a[0], a[1]));
+}
+
+// V consecutive gradient values starting at flat element index e, in fp32.
+template <int GDT, int V>
+__device__ __forceinline__ void ld_grad_v(const void *g, int64_t e, float *a) {
+    if constexpr (V == 4) {
+        to_array(ld_grad<GDT>(g, e), a);
+    } else if constexpr (GDT == MTDAO_F32) {
+        const float2 t = __ldcs(reinterpret_cast<const float2 *>(static_cast<const float *>(g) + e));
+        a[0] = t.x;
+        a[1] = t.y;
+    } else {
+        const unsigned int w =
+            __ldcs(reinterpret_cast<const unsigned int *>(static_cast<const uint16_t *>(g) + e));
+        a[0] = __uint_as_float(w << 16);
+        a[1] = __uint_as_float(w & 0xffff0000u);
+    }
+}
 
 // Writes one state's R local values (for V elements) to the lane's replicas:
 // as they are, or -- when the state is due -- all replaced by the replica
 // mean of replica_mean.cuh.  With two lane groups each group forms its part
-// of the compensated sum (replicas 1..3 and 4..7 against replica 0's value)
+// of the compensated sum (replicas 1..R-1 and R..M-1 against replica 0's
+// value; R = M / 2 is where replica_mean.cuh splits its two parts)
 // and the parts are exchanged, so both groups store exactly the value a
 // single thread would compute.  The standalone averaging kernels use the
 // same routine, so fused and separate averaging give identical bits.
@@ -68,18 +107,18 @@ __device__ __forceinline__ void store_replicas(float *state, int64_t n_padded, i
                     if (r > 0 || grp != 0) part.add(val[r][k]);
                 const float mine = part.partial();
                 const float other = __shfl_xor_sync(0xffffffffu, mine, S::kLanes);
-                const float a = grp == 0 ? mine : other;          // replicas 1 .. 3
-                const float b = grp == 0 ? other : mine;          // replicas 4 .. 7
+                const float a = grp == 0 ? mine : other;          // replicas 1 .. R-1
+                const float b = grp == 0 ? other : mine;          // replicas R .. M-1
                 mean[k] = replica_mean_from_parts(s0, a, b, static_cast<float>(M));
             }
         }
 #pragma unroll
         for (int r = 0; r < S::R; ++r)
-            st_v(state + (grp * S::R + r) * n_padded + e, mean);
+            st_v<S::V>(state + (grp * S::R + r) * n_padded + e, mean);
     } else {
 #pragma unroll
         for (int r = 0; r < S::R; ++r)
-            st_v(state + (grp * S::R + r) * n_padded + e, val[r]);
+            st_v<S::V>(state + (grp * S::R + r) * n_padded + e, val[r]);
     }
 }
 
@@ -88,7 +127,7 @@ __device__ __forceinline__ void load_replicas(const float *state, int64_t n_padd
                                               float (&val)[FusedShape<M>::R][FusedShape<M>::V]) {
     using S = FusedShape<M>;
 #pragma unroll
-    for (int r = 0; r < S::R; ++r) ld_v(state + (grp * S::R + r) * n_padded + e, val[r]);
+    for (int r = 0; r < S::R; ++r) ld_v<S::V>(state + (grp * S::R + r) * n_padded + e, val[r]);
 }
 
 template <int BASE, int N, int GDT, bool CLIP, int M>
@@ -113,7 +152,7 @@ __global__ void __launch_bounds__(kThreads, 2) step_sync_kernel(const StepArgs a
         const int64_t e = c * S::kChunk + V * q;
         float g[R][V];
 #pragma unroll
-        for (int r = 0; r < R; ++r) to_array(ld_grad<GDT>(a.grads, (grp * R + r) * n + e), g[r]);
+        for (int r = 0; r < R; ++r) ld_grad_v<GDT, V>(a.grads, (grp * R + r) * n + e, g[r]);
 
         // State by state in state_order; the next state's loads are issued
         // before the current state is updated and stored (different states
@@ -206,7 +245,9 @@ template <int BASE, int N, int GDT, bool CLIP>
 cudaError_t launch_step_sync_m(const StepArgs &a, int num_sms, cudaStream_t st) {
     switch (a.M) {
         case 2: return launch_step_sync_t<BASE, N, GDT, CLIP, 2>(a, num_sms, st);
+        case 3: return launch_step_sync_t<BASE, N, GDT, CLIP, 3>(a, num_sms, st);
         case 4: return launch_step_sync_t<BASE, N, GDT, CLIP, 4>(a, num_sms, st);
+        case 6: return launch_step_sync_t<BASE, N, GDT, CLIP, 6>(a, num_sms, st);
         case 8: return launch_step_sync_t<BASE, N, GDT, CLIP, 8>(a, num_sms, st);
         default: return cudaErrorNotSupported;
     }
