@@ -390,9 +390,16 @@ def run_ours(args):
     # end to end through the host-buffer C-ABI call
     e2e = None
     if not args.no_e2e and args.e2e_rounds > 0:
-        host_g = torch.empty((M, n), dtype=grads.dtype, pin_memory=True)
+        host_mem = "pinned"
+        try:
+            host_g = torch.empty((M, n), dtype=grads.dtype, pin_memory=True)
+        except RuntimeError:
+            # many ranks pinning tens of GB each can exhaust pinnable memory:
+            # pageable gradients go through the library's staging copy
+            host_g = torch.empty((M, n), dtype=grads.dtype)
+            host_mem = "pageable"
         host_g.copy_(grads)
-        host_x = torch.empty((n,), dtype=torch.float32, pin_memory=True)
+        host_x = torch.empty((n,), dtype=torch.float32, pin_memory=host_mem == "pinned")
         P.mtdao_step_host(eng.h, host_g.data_ptr(), gdt, opt["lr"], eng.sync_due())
         torch.cuda.synchronize()
         if dist is not None:
@@ -406,7 +413,7 @@ def run_ours(args):
         e2e_s = max_over_ranks(time.perf_counter() - t0, dist, "cuda")
         e2e = {"value": job_rate(M * n * H * args.e2e_rounds, world, e2e_s), "unit": "params/s",
                "h2d_bytes_per_step": H * M * n * g_bytes, "d2h_bytes_per_step": n * 4,
-               "rounds": args.e2e_rounds}
+               "rounds": args.e2e_rounds, "host_memory": host_mem}
         del host_g
 
     cpu = None
