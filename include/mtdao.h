@@ -238,7 +238,7 @@ int mtdao_set_params(mtdao_handle h, const float *x0_dev);
  * sync_mask: states to average over the replicas at the end of this same
  *   step (E_m[.] of Algorithm 1); usually the value of mtdao_sync_due.  The
  *   average is fused into the step's pass: it costs no extra HBM traffic for
- *   M in {2, 3, 4, 6, 8, 16}; other M fall back to a separate averaging
+ *   2 <= M <= 8 and M = 16; other M fall back to a separate averaging
  *   pass.
  * With MTDAO_CLIP_GLOBAL_NORM a reduction pass over grads precedes the step.
  * Errors: MTDAO_ERR_INVALID (dtype, mask bits beyond the states),

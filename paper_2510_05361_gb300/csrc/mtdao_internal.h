@@ -57,7 +57,7 @@ cudaError_t launch_step(int base, int n_mom, int grad_dtype, bool clip, const St
                         int num_sms, cudaStream_t stream);
 
 // Local step with the replica average of the states in a.sync_mask fused
-// into the same pass.  For M in {2, 3, 4, 6, 8, 16}; returns cudaErrorNotSupported
+// into the same pass.  For 2 <= M <= 8 and M = 16; returns cudaErrorNotSupported
 // otherwise (the caller then runs launch_step followed by launch_sync).
 cudaError_t launch_step_sync(int base, int n_mom, int grad_dtype, bool clip, const StepArgs &a,
                              int num_sms, cudaStream_t stream);

@@ -2,7 +2,7 @@
 //
 // step_sync_kernel is element-major: a lane updates the same few elements
 // of all M replicas (M = 2, 3, 4) or of a share of them while other lanes
-// of the warp hold the rest (M = 6, 8, 16; see FusedShape), with
+// of the warp hold the rest (M = 5 .. 8 and 16; see FusedShape), with
 // the update of step_kernels.cuh; then it writes each state due for
 // averaging as the replica mean (E_m[.] of Algorithms 1-3) instead of the
 // local values.  The average costs no HBM traffic beyond the step's own.
@@ -16,21 +16,21 @@ namespace mtdao {
 // ---------------------------------------------------------------- fused step + sync
 
 // Layout of the fused kernel's work.  A lane holds V consecutive elements
-// of R replicas:
+// of up to R replicas:
 //   M = 2, 3, 4 : one lane group, R = M, V = 4 (128-bit accesses);
-//   M = 6, 8    : two lane groups (half-warps), R = M / 2: lanes q and
-//                 q + 16 hold the same elements, replicas 0..R-1 and R..M-1
-//                 -- exactly the two parts of the compensated mean of
-//                 replica_mean.cuh -- and combine them by shuffles; V = 4
-//                 for M = 8, V = 2 for M = 6 (three replicas of four
-//                 elements spilled registers);
+//   M = 5 .. 8  : two lane groups (half-warps): lanes q and q + 16 hold the
+//                 same elements, replicas 0 .. M/2-1 and M/2 .. M-1 --
+//                 exactly the two parts of the compensated mean of
+//                 replica_mean.cuh -- and combine them by shuffles; for odd
+//                 M the first group has one replica fewer (its last slot
+//                 stays empty).  V = 4 for M = 8, V = 2 for M = 5, 6, 7
+//                 (four elements spilled registers);
 //   M = 16      : four lane groups of R = 4 replicas, V = 4; each part of
 //                 the mean spans two groups and its compensated sum is
 //                 handed from one to the next in replica order.
-// Other M take the plain step followed by the standalone average: 5 and 7
-// (one lane group of 5 or 7 replicas spills even at V = 2), 32 (eight
-// groups of four lanes: 64-byte pieces of eight replica slabs per load,
-// slower than the separate average) and above.
+// Other M take the plain step followed by the standalone average: 32
+// (eight groups of four lanes: 64-byte pieces of eight replica slabs per
+// load, slower than the separate average) and every M above 8 but 16.
 // The states are visited one after another (state_order); the next
 // state's loads are issued before the current state is updated and stored,
 // so two states' loads are in flight per lane within the 128-register cap.
@@ -41,13 +41,32 @@ namespace mtdao {
 // the same with or without it.
 template <int M>
 struct FusedShape {
-    static_assert(M == 2 || M == 3 || M == 4 || M == 6 || M == 8 || M == 16, "no fused shape for this M");
-    static constexpr int G = M == 16 ? 4 : (M == 6 || M == 8) ? 2 : 1;   // lane groups per warp
-    static constexpr int R = M / G;                         // replicas per lane
-    static constexpr int V = M == 6 ? 2 : 4;                // elements per lane
+    static_assert((M >= 2 && M <= 8) || M == 16, "no fused shape for this M");
+    static constexpr int G = M == 16 ? 4 : M >= 5 ? 2 : 1;     // lane groups per warp
+    // replicas of group 0 and of the other groups: with two groups the
+    // split is at M / 2, where replica_mean.cuh splits its two parts
+    static constexpr int R0 = G == 2 ? M / 2 : M / G;
+    static constexpr int R1 = G == 2 ? M - M / 2 : M / G;
+    static constexpr int R = R1;                            // replica slots per lane (R1 >= R0)
+    static constexpr bool kUniform = R0 == R1;
+    static constexpr int V = (M >= 5 && M <= 7) ? 2 : 4;  // elements per lane
     static constexpr int kLanes = 32 / G;                   // lanes per group
     static constexpr int kChunk = kLanes * V;               // elements per warp iteration
 };
+
+// First replica and number of replicas of lane group grp.
+template <int M>
+__device__ __forceinline__ int first_replica(int grp) {
+    using S = FusedShape<M>;
+    if constexpr (S::kUniform) return grp * S::R;
+    else return grp == 0 ? 0 : S::R0;
+}
+template <int M>
+__device__ __forceinline__ bool has_replica(int grp, int r) {
+    using S = FusedShape<M>;
+    if constexpr (S::kUniform) return true;
+    else return r < (grp == 0 ? S::R0 : S::R1);
+}
 
 template <int V>
 __device__ __forceinline__ void ld_v(const float *p, float *a) {
@@ -139,7 +158,7 @@ __device__ __forceinline__ void store_replicas(float *state, int64_t n_padded, i
                 DiffSum part(s0);
 #pragma unroll
                 for (int r = 0; r < S::R; ++r)      // constant indices: val stays in registers
-                    if (r > 0 || grp != 0) part.add(val[r][k]);
+                    if ((r > 0 || grp != 0) && has_replica<M>(grp, r)) part.add(val[r][k]);
                 const float mine = part.partial();
                 const float other = __shfl_xor_sync(0xffffffffu, mine, S::kLanes);
                 const float a = grp == 0 ? mine : other;          // replicas 1 .. R-1
@@ -149,11 +168,11 @@ __device__ __forceinline__ void store_replicas(float *state, int64_t n_padded, i
         }
 #pragma unroll
         for (int r = 0; r < S::R; ++r)
-            st_v<S::V>(state + (grp * S::R + r) * n_padded + e, mean);
+            if (has_replica<M>(grp, r)) st_v<S::V>(state + (first_replica<M>(grp) + r) * n_padded + e, mean);
     } else {
 #pragma unroll
         for (int r = 0; r < S::R; ++r)
-            st_v<S::V>(state + (grp * S::R + r) * n_padded + e, val[r]);
+            if (has_replica<M>(grp, r)) st_v<S::V>(state + (first_replica<M>(grp) + r) * n_padded + e, val[r]);
     }
 }
 
@@ -162,7 +181,14 @@ __device__ __forceinline__ void load_replicas(const float *state, int64_t n_padd
                                               float (&val)[FusedShape<M>::R][FusedShape<M>::V]) {
     using S = FusedShape<M>;
 #pragma unroll
-    for (int r = 0; r < S::R; ++r) ld_v<S::V>(state + (grp * S::R + r) * n_padded + e, val[r]);
+    for (int r = 0; r < S::R; ++r) {
+        if (has_replica<M>(grp, r)) {
+            ld_v<S::V>(state + (first_replica<M>(grp) + r) * n_padded + e, val[r]);
+        } else {
+#pragma unroll
+            for (int k = 0; k < S::V; ++k) val[r][k] = 0.0f;      // an empty slot of the smaller group
+        }
+    }
 }
 
 template <int BASE, int N, int GDT, bool CLIP, int M>
@@ -181,13 +207,21 @@ __global__ void __launch_bounds__(kThreads, 2) step_sync_kernel(const StepArgs a
 
     float s[R];
 #pragma unroll
-    for (int r = 0; r < R; ++r) s[r] = CLIP ? __ldg(a.clip_scale + grp * R + r) : 1.0f;
+    for (int r = 0; r < R; ++r)
+        s[r] = CLIP && has_replica<M>(grp, r) ? __ldg(a.clip_scale + first_replica<M>(grp) + r) : 1.0f;
 
     for (int64_t c = warp; c < n_chunks; c += n_warps) {
         const int64_t e = c * S::kChunk + V * q;
         float g[R][V];
 #pragma unroll
-        for (int r = 0; r < R; ++r) ld_grad_v<GDT, V>(a.grads, (grp * R + r) * n + e, g[r]);
+        for (int r = 0; r < R; ++r) {
+            if (has_replica<M>(grp, r)) {
+                ld_grad_v<GDT, V>(a.grads, (first_replica<M>(grp) + r) * n + e, g[r]);
+            } else {
+#pragma unroll
+                for (int k = 0; k < V; ++k) g[r][k] = 0.0f;
+            }
+        }
 
         // State by state in state_order; the next state's loads are issued
         // before the current state is updated and stored (different states
@@ -282,7 +316,9 @@ cudaError_t launch_step_sync_m(const StepArgs &a, int num_sms, cudaStream_t st) 
         case 2: return launch_step_sync_t<BASE, N, GDT, CLIP, 2>(a, num_sms, st);
         case 3: return launch_step_sync_t<BASE, N, GDT, CLIP, 3>(a, num_sms, st);
         case 4: return launch_step_sync_t<BASE, N, GDT, CLIP, 4>(a, num_sms, st);
+        case 5: return launch_step_sync_t<BASE, N, GDT, CLIP, 5>(a, num_sms, st);
         case 6: return launch_step_sync_t<BASE, N, GDT, CLIP, 6>(a, num_sms, st);
+        case 7: return launch_step_sync_t<BASE, N, GDT, CLIP, 7>(a, num_sms, st);
         case 8: return launch_step_sync_t<BASE, N, GDT, CLIP, 8>(a, num_sms, st);
         case 16: return launch_step_sync_t<BASE, N, GDT, CLIP, 16>(a, num_sms, st);
         default: return cudaErrorNotSupported;

@@ -71,7 +71,7 @@ RAGGED = [1, 7, 300, 4099, 2560, 13]
 @pytest.mark.parametrize("gdt", ["f32", "bf16"])
 @pytest.mark.parametrize("N", [1, 2, 3, 4])
 @pytest.mark.parametrize("base", ["adam", "adopt", "sgdm"])
-@pytest.mark.parametrize("M", [2, 3, 4, 5, 6, 8, 16, 32])
+@pytest.mark.parametrize("M", [2, 3, 4, 5, 6, 7, 8, 16, 32])
 def test_step_and_sync_parity_matrix(P, base, N, gdt, M):
     betas = W.SWEEP_BETAS[:N]
     w = workload_dict(RAGGED, M, base=base, betas=betas, beta2=0.9999 if base == "adopt" else 0.999,
@@ -96,7 +96,7 @@ def test_replica_counts(P, M):
 
 
 @pytest.mark.parametrize("gdt", ["f32", "bf16"])
-@pytest.mark.parametrize("M", [2, 3, 4, 6, 8, 16, 32])
+@pytest.mark.parametrize("M", [2, 3, 4, 5, 6, 7, 8, 16, 32])
 def test_fused_sync_is_bitwise_equal_to_separate_sync(P, M, gdt):
     for base in ("adam", "adopt", "sgdm"):
         w = workload_dict(RAGGED, M, base=base, betas=(0.9, 0.99, 0.5), px=3, pu=[2, 3, 4], pv=2,
