@@ -16,10 +16,14 @@ constexpr int kThreads = 256;        // threads per block of every streaming ker
 constexpr int kChunk = 256;          // elements per warp iteration of the local step
 constexpr int kNormThreads = 256;    // threads per block of the norm reduction
 
-// Scalars of one local step t (Algorithms 1-3).  EMAs are evaluated as
-// s + c * (target - s) with c = 1 - beta, which keeps beta's precision when
-// beta is close to 1 (the float nearest 0.9999 is 1.7e-8 away from it, the
-// float nearest 1e-4 only 2.5e-12).
+// Scalars of one local step t (Algorithms 1-3).  The decay rates enter as
+// c = 1 - beta rounded to fp32, which keeps beta's precision when beta is
+// close to 1 (the float nearest 0.9999 is 1.7e-8 away from it, the float
+// nearest 1e-4 only 2.5e-12).  A first momentum is evaluated as
+// fma(c, target, fma(-c, s, s)): beta * s is formed exactly inside the
+// inner fma and rounded once, so beta = 0 gives the target exactly however
+// large s was.  The second moment uses s + c * (g^2 - s) (g^2 - s exact
+// inside an fma).
 struct StepScalars {
     float neg_lr;                    // -eta_t
     float c1[MTDAO_MAX_MOM];         // 1 - beta_{1,j}

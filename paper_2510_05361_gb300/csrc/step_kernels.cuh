@@ -92,7 +92,8 @@ __device__ __forceinline__ float step_acc_init(const StepScalars &sc, float g, f
 //   g : raw gradient g_t^m          s : clip(g, rho) factor (1 when not clipping)
 //   cur : the state's value, updated in place
 // With st visited in state_order this is Algorithm 1 (Adam), 2 (ADOPT) or
-// 3 (SGDM) for the element; the EMAs are s + (1 - beta)(target - s).
+// 3 (SGDM) for the element; a momentum is beta * s + (1 - beta) * target
+// in the fma form described with StepScalars.
 template <int BASE, int N>
 __device__ __forceinline__ void update_state(const StepScalars &sc, int st, float g, float s, float &gt,
                                              float &acc, float &cur) {
@@ -122,7 +123,7 @@ __device__ __forceinline__ void update_state(const StepScalars &sc, int st, floa
         // momentum u_j of clip(g) (Adam, SGDM) or of ADOPT's clamped g
         const int j = st - 1;
         const float target = BASE == MTDAO_BASE_ADOPT ? gt : __fmul_rn(g, s);
-        cur = fmaf(sc.c1[j], target - cur, cur);
+        cur = fmaf(sc.c1[j], target, fmaf(-sc.c1[j], cur, cur));
         acc = fmaf(sc.k[j], cur, acc);
     }
 }

@@ -290,7 +290,7 @@ __global__ void __launch_bounds__(kThreads, 2) step_sync_kernel(const StepArgs a
                     for (int k = 0; k < V; ++k) {
                         const float target =
                             BASE == MTDAO_BASE_ADOPT ? gt[r][k] : __fmul_rn(g[r][k], s[r]);
-                        cur[r][k] = fmaf(a.sc.c1[j], target - cur[r][k], cur[r][k]);
+                        cur[r][k] = fmaf(a.sc.c1[j], target, fmaf(-a.sc.c1[j], cur[r][k], cur[r][k]));
                         acc[r][k] = fmaf(a.sc.k[j], cur[r][k], acc[r][k]);
                     }
             }
