@@ -22,8 +22,8 @@ constexpr int kNormThreads = 256;    // threads per block of the norm reduction
 // nearest 1e-4 only 2.5e-12).  A first momentum is evaluated as
 // fma(c, target, fma(-c, s, s)): beta * s is formed exactly inside the
 // inner fma and rounded once, so beta = 0 gives the target exactly however
-// large s was.  The second moment uses s + c * (g^2 - s) (g^2 - s exact
-// inside an fma).
+// large s was.  The second moment is fma(c * g, g, fma(-c, s, s)) in the
+// same way, so beta_2 = 0 gives g^2.
 struct StepScalars {
     float neg_lr;                    // -eta_t
     float c1[MTDAO_MAX_MOM];         // 1 - beta_{1,j}

@@ -92,8 +92,8 @@ __device__ __forceinline__ float step_acc_init(const StepScalars &sc, float g, f
 //   g : raw gradient g_t^m          s : clip(g, rho) factor (1 when not clipping)
 //   cur : the state's value, updated in place
 // With st visited in state_order this is Algorithm 1 (Adam), 2 (ADOPT) or
-// 3 (SGDM) for the element; a momentum is beta * s + (1 - beta) * target
-// in the fma form described with StepScalars.
+// 3 (SGDM) for the element; every EMA is beta * s + (1 - beta) * target in
+// the fma form described with StepScalars.
 template <int BASE, int N>
 __device__ __forceinline__ void update_state(const StepScalars &sc, int st, float g, float s, float &gt,
                                              float &acc, float &cur) {
@@ -104,9 +104,9 @@ __device__ __forceinline__ void update_state(const StepScalars &sc, int st, floa
         float gn;
         if (sc.prev_v) {
             gn = g / (sqrtf(cur) + sc.eps);
-            cur = fmaf(sc.c2, fmaf(g, g, -cur), cur);
+            cur = fmaf(__fmul_rn(sc.c2, g), g, fmaf(-sc.c2, cur, cur));
         } else {
-            cur = fmaf(sc.c2, fmaf(g, g, -cur), cur);
+            cur = fmaf(__fmul_rn(sc.c2, g), g, fmaf(-sc.c2, cur, cur));
             gn = g / (sqrtf(cur) + sc.eps);
         }
         gn = gn > sc.clip_c ? sc.clip_c : (gn < -sc.clip_c ? -sc.clip_c : gn);  // keeps NaN
@@ -115,7 +115,7 @@ __device__ __forceinline__ void update_state(const StepScalars &sc, int st, floa
     } else if (st == 1 + N) {
         // Algorithm 1: v of the raw gradient, then the denominator
         // sqrt(v / b_v) + eps of the momenta's combination.
-        cur = fmaf(sc.c2, fmaf(g, g, -cur), cur);
+        cur = fmaf(__fmul_rn(sc.c2, g), g, fmaf(-sc.c2, cur, cur));
         acc = acc / fmaf(sqrtf(cur), sc.sv, sc.eps);
     } else if (st == 0) {
         cur = fmaf(sc.neg_lr, acc, cur);                     // x - eta_t Delta

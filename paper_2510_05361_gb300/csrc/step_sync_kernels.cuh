@@ -258,9 +258,9 @@ __global__ void __launch_bounds__(kThreads, 2) step_sync_kernel(const StepArgs a
                         float gn;
                         if (a.sc.prev_v) {
                             gn = gr / (sqrtf(cur[r][k]) + a.sc.eps);
-                            cur[r][k] = fmaf(a.sc.c2, fmaf(gr, gr, -cur[r][k]), cur[r][k]);
+                            cur[r][k] = fmaf(__fmul_rn(a.sc.c2, gr), gr, fmaf(-a.sc.c2, cur[r][k], cur[r][k]));
                         } else {
-                            cur[r][k] = fmaf(a.sc.c2, fmaf(gr, gr, -cur[r][k]), cur[r][k]);
+                            cur[r][k] = fmaf(__fmul_rn(a.sc.c2, gr), gr, fmaf(-a.sc.c2, cur[r][k], cur[r][k]));
                             gn = gr / (sqrtf(cur[r][k]) + a.sc.eps);
                         }
                         gn = gn > a.sc.clip_c ? a.sc.clip_c : (gn < -a.sc.clip_c ? -a.sc.clip_c : gn);
@@ -274,7 +274,7 @@ __global__ void __launch_bounds__(kThreads, 2) step_sync_kernel(const StepArgs a
 #pragma unroll
                     for (int k = 0; k < V; ++k) {
                         const float gr = g[r][k];
-                        cur[r][k] = fmaf(a.sc.c2, fmaf(gr, gr, -cur[r][k]), cur[r][k]);
+                        cur[r][k] = fmaf(__fmul_rn(a.sc.c2, gr), gr, fmaf(-a.sc.c2, cur[r][k], cur[r][k]));
                         acc[r][k] = acc[r][k] / fmaf(sqrtf(cur[r][k]), a.sc.sv, a.sc.eps);
                     }
             } else if (st == 0) {

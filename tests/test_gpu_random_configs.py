@@ -1,6 +1,8 @@
 """Seeded random configurations, GPU against the oracle: base, number of
-momenta, decay rates and weights (including beta = 0 and weights that sum
-to 1), periods (including 0 = never), both sync phases, clipping modes,
+momenta, decay rates and weights (including beta_1 = 0, beta_2 = 0 and
+weights that sum to 1), epsilon from 1e-12 to 1e-3, learning rates from 0
+to 0.1, gradient scales from 1e-6 to 100, periods (including 0 = never),
+both sync phases, clipping modes,
 the ADOPT ordering flag, gradient dtype and kind, the replica count and a
 ragged tensor list (with zero-size tensors) are drawn per case; every
 element of every state is compared after T steps."""
@@ -30,7 +32,7 @@ def draw(case):
     rng = np.random.default_rng(1000 + case)
     base = ["adam", "adopt", "sgdm"][case % 3]
     N = int(rng.integers(1, 5))
-    betas = [float(rng.choice([0.0, 0.5, 0.9, 0.95, 0.99, 0.999, 0.9999])) for _ in range(N)]
+    betas = [float(rng.choice([0.0, 0.1, 0.5, 0.9, 0.95, 0.99, 0.999, 0.9999])) for _ in range(N)]
     if rng.random() < 0.25:
         omega = list(rng.dirichlet(np.ones(N)))                      # sum to 1: no gradient term
         omega = [float(o) * (1 - 1e-9) for o in omega]
@@ -42,22 +44,23 @@ def draw(case):
         clip = "elementwise"
     if base != "adopt" and rng.random() < 0.3:
         clip = "global_norm"
-    M = int(rng.choice([1, 2, 3, 4, 5, 6, 7, 8, 9, 16]))
+    M = int(rng.choice([1, 2, 3, 4, 5, 6, 7, 8, 9, 12, 16, 32]))
     shapes = [int(rng.choice([0, 1, 7, 64, 333, 1000, 4099])) for _ in range(int(rng.integers(1, 6)))]
     if sum(shapes) == 0:
         shapes.append(513)
     opt = {"base": base, "n_mom": N, "beta1": betas, "omega": omega,
-           "beta2": float(rng.choice([0.99, 0.999, 0.9999])), "eps": float(rng.choice([1e-8, 1e-6])),
+           "beta2": float(rng.choice([0.0, 0.5, 0.99, 0.999, 0.9999])),
+           "eps": float(rng.choice([1e-12, 1e-8, 1e-6, 1e-3])),
            "bias_correction": base == "adam" and bool(rng.random() < 0.7), "clip_mode": clip,
            "clip_rho": float(rng.choice([0.5, 1.0, 50.0])), "period_x": periods(),
            "period_u": [periods() for _ in range(N)], "period_v": periods(),
            "sync_phase": "alg2_literal" if rng.random() < 0.3 else "alg1",
            "adopt_prev_v": base == "adopt" and bool(rng.random() < 0.4),
-           "lr": float(rng.choice([1e-3, 2.0 ** -8, 1e-2]))}
+           "lr": float(rng.choice([0.0, 1e-4, 1e-3, 2.0 ** -8, 1e-2, 0.1]))}
     w = {"name": "random", "shapes": shapes, "M": M, "grad_kind": str(rng.choice(G.KINDS)),
-         "grad_sigma": float(rng.choice([1e-3, 0.01, 1.0])),
+         "grad_sigma": float(rng.choice([1e-6, 1e-3, 0.01, 1.0, 100.0])),
          "grad_dtype": "bf16" if rng.random() < 0.4 else "f32", "init_sigma": 0.02, "opt": opt}
-    return w, int(rng.integers(3, 13))
+    return w, int(rng.integers(3, 17))
 
 
 @pytest.mark.parametrize("case", range(96))
