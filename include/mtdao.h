@@ -278,8 +278,9 @@ int mtdao_step_host(mtdao_handle h, const void *grads_host, int32_t grad_dtype, 
  * mean over the M replicas.  Computed in fp32 as s_0 + (A + B) / M, A and
  * B the Kahan-compensated sums of (s_m - s_0) over replicas 1..h-1 and
  * h..M-1 (h = floor(M/2)), each in replica order; this returns s_0 bit for
- * bit when the replicas agree and stays within about one rounding of the
- * exact mean for any M.  The fused average in mtdao_step and
+ * bit when the replicas agree, and otherwise stays within a few roundings
+ * of the largest replica value for any M (relative to the mean itself only
+ * when the replicas do not cancel).  The fused average in mtdao_step and
  * mtdao_sync_stats use the same routine (identical bits).  mask 0 is a
  * no-op.
  */
