@@ -455,6 +455,7 @@ def run_ours(args):
                              "launches_per_round": len(sync_steps) // args.steps},
         "sync_kernel": {"ms_median": statistics.median(sync_ms), "ms_min": min(sync_ms),
                         "launches": len(sync_ms), "bytes": sync_bytes, "gbs": sync_gbs,
+                        "frac_of_nominal": sync_gbs / NOMINAL_HBM_GBS,
                         "frac": sync_gbs / peak, "states": n_states},
         "sync_stats_kernel": ({"ms_median": statistics.median(stats_ms), "ms_min": min(stats_ms),
                                "gbs": sync_bytes / (statistics.median(stats_ms) / 1e3) / 1e9,
