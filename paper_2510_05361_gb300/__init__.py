@@ -361,7 +361,29 @@ class MTDAO:
     def _ptr(t) -> int:
         return t if isinstance(t, int) else int(t.data_ptr())
 
+    def _check_tensor(self, t, what: str, shape, dtypes, device: str) -> None:
+        """Tensors are passed as raw pointers, so their layout must be the
+        one the library reads: the given shape, one of the dtypes,
+        contiguous, on the given kind of device.  Raw integer pointers
+        are passed through unchecked."""
+        if isinstance(t, int):
+            return
+        if tuple(t.shape) != tuple(shape) and not (len(shape) == 1 and t.numel() == shape[0] and t.dim() == 1):
+            raise ValueError("%s: expected shape %s, got %s" % (what, tuple(shape), tuple(t.shape)))
+        if t.dtype not in dtypes:
+            raise ValueError("%s: dtype %s not supported" % (what, t.dtype))
+        if not t.is_contiguous():
+            raise ValueError("%s must be contiguous" % what)
+        if (t.device.type == "cuda") != (device == "cuda"):
+            raise ValueError("%s must be in %s memory" % (what, "device" if device == "cuda" else "host"))
+
+    def _grad_dtypes(self):
+        import torch
+        return (torch.float32, torch.bfloat16)
+
     def set_params(self, x0) -> None:
+        import torch
+        self._check_tensor(x0, "x0", (self.n_padded,), (torch.float32,), "cuda")
         mtdao_set_params(self.h, self._ptr(x0))
 
     def step(self, grads, lr: float, sync_mask: int | None = None, dtype: int | None = None) -> int:
@@ -369,6 +391,7 @@ class MTDAO:
         Returns the sync mask that was applied."""
         if sync_mask is None:
             sync_mask = mtdao_sync_due(self.h)
+        self._check_tensor(grads, "grads", (self.M, self.n_padded), self._grad_dtypes(), "cuda")
         if dtype is None:
             import torch
             dtype = BF16 if grads.dtype == torch.bfloat16 else F32
@@ -379,6 +402,7 @@ class MTDAO:
                   dtype: int | None = None) -> int:
         if sync_mask is None:
             sync_mask = mtdao_sync_due(self.h)
+        self._check_tensor(grads_host, "grads_host", (self.M, self.n_padded), self._grad_dtypes(), "cpu")
         if dtype is None:
             import torch
             dtype = BF16 if grads_host.dtype == torch.bfloat16 else F32
@@ -389,6 +413,9 @@ class MTDAO:
         """len(lrs) local steps in one call.  grads: a [count][M][n_padded]
         tensor (one buffer per step) or a [M][n_padded] tensor reused by
         every step."""
+        if not isinstance(grads, int):
+            shape = (len(lrs), self.M, self.n_padded) if grads.dim() == 3 else (self.M, self.n_padded)
+            self._check_tensor(grads, "grads", shape, self._grad_dtypes(), "cuda")
         if dtype is None:
             import torch
             dtype = BF16 if grads.dtype == torch.bfloat16 else F32

@@ -481,6 +481,31 @@ def test_handle_streams_are_respected(P):
         eng.close()
 
 
+def test_binding_rejects_tensors_the_library_would_misread(P):
+    """The library reads raw pointers, so the binding checks each tensor's
+    shape, dtype, contiguity and device before passing it on."""
+    w = workload_dict(RAGGED, 4)
+    eng = P.MTDAO(w["opt"], 4, w["shapes"])
+    n = eng.n_padded
+    good = torch.zeros((4, n), device="cuda")
+    eng.step(good, 1e-3)
+    bad = [torch.zeros((4, n - 8), device="cuda"),                 # wrong shape
+           torch.zeros((n, 4), device="cuda").t(),                 # transposed view: not contiguous
+           torch.zeros((4, n), device="cuda", dtype=torch.float16),
+           torch.zeros((4, n))]                                     # host memory for the device call
+    for g in bad:
+        with pytest.raises(ValueError):
+            eng.step(g, 1e-3)
+    with pytest.raises(ValueError):
+        eng.step_host(good, 1e-3)                                  # device memory for the host call
+    with pytest.raises(ValueError):
+        eng.set_params(torch.zeros(n + 1, device="cuda"))
+    with pytest.raises(ValueError):
+        eng.run(torch.zeros((3, 4, n), device="cuda"), [1e-3] * 2)  # count does not match lrs
+    assert eng.t == 1                                              # nothing ran
+    eng.close()
+
+
 @pytest.mark.parametrize("case", ["qhm_beta0_no_grad_term", "omega0", "sgdm_sum_omega1",
                                   "adopt_beta0", "max_replicas"])
 def test_degenerate_hyperparameters(P, case):
