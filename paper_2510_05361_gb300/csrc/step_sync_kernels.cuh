@@ -1,11 +1,11 @@
 // step_sync_kernels.cuh -- the local step with the replica average fused in.
 //
 // step_sync_kernel is element-major: a lane updates the same few elements
-// of all M replicas (M = 2, 3, 4) or of a share of them while other lanes
-// of the warp hold the rest (M = 5 .. 8 and 16; see FusedShape), with
-// the update of step_kernels.cuh; then it writes each state due for
-// averaging as the replica mean (E_m[.] of Algorithms 1-3) instead of the
-// local values.  The average costs no HBM traffic beyond the step's own.
+// of all M replicas (M <= 7) or of a share of them while other lanes of the
+// warp hold the rest (M = 8 and 16; see FusedShape), with the update of
+// step_kernels.cuh; then it writes each state due for averaging as the
+// replica mean (E_m[.] of Algorithms 1-3) instead of the local values.  The
+// average costs no HBM traffic beyond the step's own.
 #pragma once
 
 #include "replica_mean.cuh"
@@ -16,57 +16,37 @@ namespace mtdao {
 // ---------------------------------------------------------------- fused step + sync
 
 // Layout of the fused kernel's work.  A lane holds V consecutive elements
-// of up to R replicas:
-//   M = 2, 3, 4 : one lane group, R = M, V = 4 (128-bit accesses);
-//   M = 5 .. 8  : two lane groups (half-warps): lanes q and q + 16 hold the
-//                 same elements, replicas 0 .. M/2-1 and M/2 .. M-1 --
-//                 exactly the two parts of the compensated mean of
-//                 replica_mean.cuh -- and combine them by shuffles; for odd
-//                 M the first group has one replica fewer (its last slot
-//                 stays empty).  V = 4 for M = 8, V = 2 for M = 5, 6, 7
-//                 (four elements spilled registers);
-//   M = 16      : four lane groups of R = 4 replicas, V = 4; each part of
-//                 the mean spans two groups and its compensated sum is
-//                 handed from one to the next in replica order.
+// of R replicas; the G lane groups of a warp hold the same elements of
+// different replicas (group k: replicas k*R .. k*R + R-1):
+//   M = 2, 3, 4 : one group, R = M, V = 4 (128-bit accesses);
+//   M = 5, 6, 7 : one group, R = M, V = 2 (four elements spill registers);
+//   M = 8       : two groups (half-warps) of R = 4, V = 4: replicas 0..3 and
+//                 4..7 are the two parts of the compensated mean of
+//                 replica_mean.cuh, combined by one shuffle;
+//   M = 16      : four groups of R = 4, V = 4; each part of the mean spans
+//                 two groups and its compensated sum is handed from one to
+//                 the next in replica order.
 // Other M take the plain step followed by the standalone average: 32
 // (eight groups of four lanes: 64-byte pieces of eight replica slabs per
 // load, slower than the separate average) and every M above 8 but 16.
 // The states are visited one after another (state_order); the next
 // state's loads are issued before the current state is updated and stored,
 // so two states' loads are in flight per lane within the 128-register cap.
-// Measured on the flat 2^27 sweep (GB/s of the fused step, Adam, f32): the
-// lookahead lifts M = 8 from 6030-6065 to 6485-6727 (ADOPT with bf16
-// gradients: 5439 -> 6089) and M = 4 from 6413-6556 (2 elements per lane,
-// every load of the chunk first, as in step_kernel) to 6582-6718; M = 2 is
-// the same with or without it.
+// What a warp keeps in flight sets the pace: M = 5..7 as two half-warp
+// groups of V = 2 (half the bytes per warp) ran the fused step at
+// 3.7-5.8 TB/s on the flat 2^27 sweep, as one group 5.8-6.7 TB/s.  The
+// lookahead lifted M = 8 from 6030-6065 GB/s to 6485-6727 and M = 4 from
+// 6413-6556 (2 elements per lane, every load of the chunk first, as in
+// step_kernel) to 6582-6718; M = 2 is the same with or without it.
 template <int M>
 struct FusedShape {
     static_assert((M >= 2 && M <= 8) || M == 16, "no fused shape for this M");
-    static constexpr int G = M == 16 ? 4 : M >= 5 ? 2 : 1;     // lane groups per warp
-    // replicas of group 0 and of the other groups: with two groups the
-    // split is at M / 2, where replica_mean.cuh splits its two parts
-    static constexpr int R0 = G == 2 ? M / 2 : M / G;
-    static constexpr int R1 = G == 2 ? M - M / 2 : M / G;
-    static constexpr int R = R1;                            // replica slots per lane (R1 >= R0)
-    static constexpr bool kUniform = R0 == R1;
-    static constexpr int V = (M >= 5 && M <= 7) ? 2 : 4;  // elements per lane
-    static constexpr int kLanes = 32 / G;                   // lanes per group
-    static constexpr int kChunk = kLanes * V;               // elements per warp iteration
+    static constexpr int G = M == 16 ? 4 : M == 8 ? 2 : 1;    // lane groups per warp
+    static constexpr int R = M / G;                          // replicas per lane
+    static constexpr int V = (M >= 5 && M <= 7) ? 2 : 4;     // elements per lane
+    static constexpr int kLanes = 32 / G;                    // lanes per group
+    static constexpr int kChunk = kLanes * V;                // elements per warp iteration
 };
-
-// First replica and number of replicas of lane group grp.
-template <int M>
-__device__ __forceinline__ int first_replica(int grp) {
-    using S = FusedShape<M>;
-    if constexpr (S::kUniform) return grp * S::R;
-    else return grp == 0 ? 0 : S::R0;
-}
-template <int M>
-__device__ __forceinline__ bool has_replica(int grp, int r) {
-    using S = FusedShape<M>;
-    if constexpr (S::kUniform) return true;
-    else return r < (grp == 0 ? S::R0 : S::R1);
-}
 
 template <int V>
 __device__ __forceinline__ void ld_v(const float *p, float *a) {
@@ -158,7 +138,7 @@ __device__ __forceinline__ void store_replicas(float *state, int64_t n_padded, i
                 DiffSum part(s0);
 #pragma unroll
                 for (int r = 0; r < S::R; ++r)      // constant indices: val stays in registers
-                    if ((r > 0 || grp != 0) && has_replica<M>(grp, r)) part.add(val[r][k]);
+                    if (r > 0 || grp != 0) part.add(val[r][k]);
                 const float mine = part.partial();
                 const float other = __shfl_xor_sync(0xffffffffu, mine, S::kLanes);
                 const float a = grp == 0 ? mine : other;          // replicas 1 .. R-1
@@ -168,11 +148,11 @@ __device__ __forceinline__ void store_replicas(float *state, int64_t n_padded, i
         }
 #pragma unroll
         for (int r = 0; r < S::R; ++r)
-            if (has_replica<M>(grp, r)) st_v<S::V>(state + (first_replica<M>(grp) + r) * n_padded + e, mean);
+            st_v<S::V>(state + (grp * S::R + r) * n_padded + e, mean);
     } else {
 #pragma unroll
         for (int r = 0; r < S::R; ++r)
-            if (has_replica<M>(grp, r)) st_v<S::V>(state + (first_replica<M>(grp) + r) * n_padded + e, val[r]);
+            st_v<S::V>(state + (grp * S::R + r) * n_padded + e, val[r]);
     }
 }
 
@@ -181,14 +161,7 @@ __device__ __forceinline__ void load_replicas(const float *state, int64_t n_padd
                                               float (&val)[FusedShape<M>::R][FusedShape<M>::V]) {
     using S = FusedShape<M>;
 #pragma unroll
-    for (int r = 0; r < S::R; ++r) {
-        if (has_replica<M>(grp, r)) {
-            ld_v<S::V>(state + (first_replica<M>(grp) + r) * n_padded + e, val[r]);
-        } else {
-#pragma unroll
-            for (int k = 0; k < S::V; ++k) val[r][k] = 0.0f;      // an empty slot of the smaller group
-        }
-    }
+    for (int r = 0; r < S::R; ++r) ld_v<S::V>(state + (grp * S::R + r) * n_padded + e, val[r]);
 }
 
 template <int BASE, int N, int GDT, bool CLIP, int M>
@@ -208,20 +181,23 @@ __global__ void __launch_bounds__(kThreads, 2) step_sync_kernel(const StepArgs a
     float s[R];
 #pragma unroll
     for (int r = 0; r < R; ++r)
-        s[r] = CLIP && has_replica<M>(grp, r) ? __ldg(a.clip_scale + first_replica<M>(grp) + r) : 1.0f;
+        s[r] = CLIP ? __ldg(a.clip_scale + grp * R + r) : 1.0f;
 
     for (int64_t c = warp; c < n_chunks; c += n_warps) {
         const int64_t e = c * S::kChunk + V * q;
+        // Left to itself ptxas keeps the address of every (state, replica)
+        // slab in registers across the loop and, with bf16 gradients or
+        // V = 2, spills (M = 8, ADOPT, N = 2, bf16: 128 registers and an
+        // 8-byte spill).  Passing the two strides through an empty asm
+        // statement each iteration makes it recompute the addresses
+        // instead (120 registers, no spill; the fused step of that case
+        // from 6063 to 6563 GB/s on a flat 2^27).  The f32 instances
+        // fit without it and run as fast.
+        int64_t nn = n, stride = a.stride;
+        if constexpr (GDT == MTDAO_BF16 || V == 2) asm volatile("" : "+l"(nn), "+l"(stride));
         float g[R][V];
 #pragma unroll
-        for (int r = 0; r < R; ++r) {
-            if (has_replica<M>(grp, r)) {
-                ld_grad_v<GDT, V>(a.grads, (first_replica<M>(grp) + r) * n + e, g[r]);
-            } else {
-#pragma unroll
-                for (int k = 0; k < V; ++k) g[r][k] = 0.0f;
-            }
-        }
+        for (int r = 0; r < R; ++r) ld_grad_v<GDT, V>(a.grads, (grp * R + r) * nn + e, g[r]);
 
         // State by state in state_order; the next state's loads are issued
         // before the current state is updated and stored (different states
@@ -243,9 +219,9 @@ __global__ void __launch_bounds__(kThreads, 2) step_sync_kernel(const StepArgs a
         for (int i = 0; i < kStates; ++i) {
             const int st = state_order<BASE, N>(i);
             if (i == 0)
-                load_replicas<M>(a.arena + st * a.stride, n, e, grp, buf[0]);
+                load_replicas<M>(a.arena + st * stride, nn, e, grp, buf[0]);
             if (i + 1 < kStates)
-                load_replicas<M>(a.arena + state_order<BASE, N>(i + 1) * a.stride, n, e, grp,
+                load_replicas<M>(a.arena + state_order<BASE, N>(i + 1) * stride, nn, e, grp,
                                  buf[(i + 1) & 1]);
             float (&cur)[R][V] = buf[i & 1];
             if (st == 1 + N && BASE == MTDAO_BASE_ADOPT) {
@@ -294,7 +270,7 @@ __global__ void __launch_bounds__(kThreads, 2) step_sync_kernel(const StepArgs a
                         acc[r][k] = fmaf(a.sc.k[j], cur[r][k], acc[r][k]);
                     }
             }
-            store_replicas<M>(a.arena + st * a.stride, n, e, grp, cur, (mask >> st) & 1u);
+            store_replicas<M>(a.arena + st * stride, nn, e, grp, cur, (mask >> st) & 1u);
         }
     }
 }
