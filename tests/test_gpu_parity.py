@@ -110,7 +110,7 @@ def test_fused_sync_is_bitwise_equal_to_separate_sync(P, M, gdt):
         b.close()
 
 
-@pytest.mark.parametrize("M", [3, 4, 8])
+@pytest.mark.parametrize("M", [3, 4, 5, 7, 8, 16])
 @pytest.mark.parametrize("gdt", ["f32", "bf16"])
 @pytest.mark.parametrize("base", ["adam", "sgdm"])
 def test_global_norm_clip_parity(P, base, gdt, M):
