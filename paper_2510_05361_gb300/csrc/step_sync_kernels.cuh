@@ -22,7 +22,7 @@ namespace mtdao {
 //   M = 5, 6, 7 : one group, R = M, V = 2 (four elements spill registers);
 //   M = 8       : two groups (half-warps) of R = 4, V = 4: replicas 0..3 and
 //                 4..7 are the two parts of the compensated mean of
-//                 replica_mean.cuh, combined by one shuffle;
+//                 replica_mean.cuh, combined by shuffles;
 //   M = 16      : four groups of R = 4, V = 4; each part of the mean spans
 //                 two groups and its compensated sum is handed from one to
 //                 the next in replica order.
@@ -32,9 +32,9 @@ namespace mtdao {
 // The states are visited one after another (state_order); the next
 // state's loads are issued before the current state is updated and stored,
 // so two states' loads are in flight per lane within the 128-register cap.
-// What a warp keeps in flight sets the pace: M = 5..7 as two half-warp
-// groups of V = 2 (half the bytes per warp) ran the fused step at
-// 3.7-5.8 TB/s on the flat 2^27 sweep, as one group 5.8-6.7 TB/s.  The
+// Holding all replicas in one lane doubled the bytes a warp of M = 5..7
+// has in flight: as two half-warp groups of V = 2 they ran the fused step
+// at 3.7-5.8 TB/s on the flat 2^27 sweep, as one group at 5.8-6.7.  The
 // lookahead lifted M = 8 from 6030-6065 GB/s to 6485-6727 and M = 4 from
 // 6413-6556 (2 elements per lane, every load of the chunk first, as in
 // step_kernel) to 6582-6718; M = 2 is the same with or without it.
