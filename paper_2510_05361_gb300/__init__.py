@@ -381,6 +381,19 @@ class MTDAO:
         import torch
         return (torch.float32, torch.bfloat16)
 
+    @staticmethod
+    def _grad_code(grads, dtype):
+        """The library's dtype code for a gradient buffer: the tensor's own
+        (an explicit dtype must agree with it); for a raw pointer the given
+        dtype, else F32."""
+        if isinstance(grads, int):
+            return F32 if dtype is None else dtype
+        import torch
+        code = BF16 if grads.dtype == torch.bfloat16 else F32
+        if dtype is not None and dtype != code:
+            raise ValueError("dtype %d does not match the gradient tensor's %s" % (dtype, grads.dtype))
+        return code
+
     def set_params(self, x0) -> None:
         import torch
         self._check_tensor(x0, "x0", (self.n_padded,), (torch.float32,), "cuda")
@@ -392,9 +405,7 @@ class MTDAO:
         if sync_mask is None:
             sync_mask = mtdao_sync_due(self.h)
         self._check_tensor(grads, "grads", (self.M, self.n_padded), self._grad_dtypes(), "cuda")
-        if dtype is None:
-            import torch
-            dtype = BF16 if grads.dtype == torch.bfloat16 else F32
+        dtype = self._grad_code(grads, dtype)
         mtdao_step(self.h, self._ptr(grads), dtype, lr, sync_mask)
         return sync_mask
 
@@ -403,23 +414,19 @@ class MTDAO:
         if sync_mask is None:
             sync_mask = mtdao_sync_due(self.h)
         self._check_tensor(grads_host, "grads_host", (self.M, self.n_padded), self._grad_dtypes(), "cpu")
-        if dtype is None:
-            import torch
-            dtype = BF16 if grads_host.dtype == torch.bfloat16 else F32
+        dtype = self._grad_code(grads_host, dtype)
         mtdao_step_host(self.h, self._ptr(grads_host), dtype, lr, sync_mask)
         return sync_mask
 
     def run(self, grads, lrs, dtype: int | None = None) -> None:
         """len(lrs) local steps in one call.  grads: a [count][M][n_padded]
-        tensor (one buffer per step) or a [M][n_padded] tensor reused by
-        every step."""
-        if not isinstance(grads, int):
-            shape = (len(lrs), self.M, self.n_padded) if grads.dim() == 3 else (self.M, self.n_padded)
-            self._check_tensor(grads, "grads", shape, self._grad_dtypes(), "cuda")
-        if dtype is None:
-            import torch
-            dtype = BF16 if grads.dtype == torch.bfloat16 else F32
-        stride = grads.stride(0) * grads.element_size() if grads.dim() == 3 else 0
+        tensor (one buffer per step) or a [M][n_padded] tensor (or a raw
+        device pointer to one) reused by every step."""
+        three_d = not isinstance(grads, int) and grads.dim() == 3
+        shape = (len(lrs), self.M, self.n_padded) if three_d else (self.M, self.n_padded)
+        self._check_tensor(grads, "grads", shape, self._grad_dtypes(), "cuda")
+        dtype = self._grad_code(grads, dtype)
+        stride = grads.stride(0) * grads.element_size() if three_d else 0
         mtdao_run(self.h, self._ptr(grads), stride, dtype, lrs)
 
     def sync(self, mask: int) -> None:

@@ -168,3 +168,20 @@ def test_half_life_helpers_reject_bad_arguments(P):
     cfg.period_v = -3
     with pytest.raises(P.MTDAOError):
         P.mtdao_comm_reduction(cfg)
+
+
+def test_binding_gradient_dtype_code(P):
+    """The binding derives the library's dtype code from the gradient
+    tensor and refuses an explicit code that contradicts it (the kernel
+    would read the buffer as the other type)."""
+    import torch
+    code = P.MTDAO._grad_code
+    assert code(torch.zeros(3), None) == P.F32
+    assert code(torch.zeros(3, dtype=torch.bfloat16), None) == P.BF16
+    assert code(torch.zeros(3, dtype=torch.bfloat16), P.BF16) == P.BF16
+    assert code(0x1000, None) == P.F32              # a raw pointer: as given, F32 by default
+    assert code(0x1000, P.BF16) == P.BF16
+    with pytest.raises(ValueError):
+        code(torch.zeros(3), P.BF16)
+    with pytest.raises(ValueError):
+        code(torch.zeros(3, dtype=torch.bfloat16), P.F32)

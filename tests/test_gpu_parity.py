@@ -497,6 +497,8 @@ def test_binding_rejects_tensors_the_library_would_misread(P):
         with pytest.raises(ValueError):
             eng.step(g, 1e-3)
     with pytest.raises(ValueError):
+        eng.step(good, 1e-3, dtype=P.BF16)                         # code contradicts the tensor
+    with pytest.raises(ValueError):
         eng.step_host(good, 1e-3)                                  # device memory for the host call
     with pytest.raises(ValueError):
         eng.set_params(torch.zeros(n + 1, device="cuda"))
