@@ -1,10 +1,10 @@
 // step_kernels.cuh -- the MT-DAO local step (Algorithms 1-3) for sm_103a.
 //
 // The step is elementwise and HBM-bound (about 0.3 flop per byte), so it is
-// written as a persistent grid-stride streaming kernel: every state of every
-// replica is read once and written once per step with 128-bit accesses, the
-// gradient is read once.  A warp owns a chunk of 256 consecutive elements
-// per iteration; lane l handles elements [4l, 4l+4) and [128+4l, 128+4l+4)
+// written as a grid-stride streaming kernel launched with one chunk per
+// warp (stream_grid): every state of every replica is read once and written
+// once per step with 128-bit accesses, the gradient is read once.  A warp
+// owns a chunk of 256 consecutive elements; lane l handles elements [4l, 4l+4) and [128+4l, 128+4l+4)
 // of the chunk, so every warp-wide load or store instruction covers 512
 // contiguous bytes of fp32 (256 bytes of bf16 gradient).
 //
@@ -198,11 +198,25 @@ inline int persistent_grid(int per_sm, int num_sms, int64_t n_warp_items) {
     return static_cast<int>(grid < 1 ? 1 : grid);
 }
 
+// Streaming grid: one warp chunk per warp, so the loop of the kernel runs
+// once (it stays a grid-stride loop, so any grid is correct).  The block
+// scheduler starts blocks in index order as earlier ones retire, which
+// keeps the addresses in flight within a narrow window of every slab; a
+// persistent grid's warps drift apart over the whole slab.  On the ~1B
+// and ~350M workloads the local step ran 10-12% faster this way (7158 vs
+// 6484 GB/s, 7128 vs 6375 GB/s on one box).
+inline int stream_grid(int64_t n_warp_items) {
+    const int64_t warps_per_block = kThreads / 32;
+    int64_t grid = (n_warp_items + warps_per_block - 1) / warps_per_block;
+    if (grid > 0x7fffffff) grid = 0x7fffffff;
+    return static_cast<int>(grid < 1 ? 1 : grid);
+}
+
 template <int BASE, int N, int GDT, bool CLIP>
 cudaError_t launch_step_t(const StepArgs &a, int num_sms, cudaStream_t stream) {
     auto kernel = step_kernel<BASE, N, GDT, CLIP>;
-    static const int per_sm = blocks_per_sm(kernel);
-    const int grid = persistent_grid(per_sm, num_sms, a.stride / kChunk);
+    (void)num_sms;
+    const int grid = stream_grid(a.stride / kChunk);
     kernel<<<grid, kThreads, 0, stream>>>(a);
     return cudaGetLastError();
 }

@@ -279,9 +279,22 @@ __global__ void __launch_bounds__(kThreads, 2) step_sync_kernel(const StepArgs a
 
 template <int BASE, int N, int GDT, bool CLIP, int M>
 cudaError_t launch_step_sync_t(const StepArgs &a, int num_sms, cudaStream_t stream) {
+    // One chunk per warp (stream_grid) where a warp's chunk spans 128
+    // elements or more (M <= 4), except for Adam and ADOPT with a single
+    // momentum.  Measured on flat 2^27 cases (GB/s, persistent -> one chunk
+    // per warp): the ~1B workload's fused step (M = 4, N = 3) 6510 -> 6964,
+    // M = 4 N = 2..4 6.6 -> 6.9-7.0 TB/s, SGDM N = 1 6487 -> 7061, but Adam
+    // N = 1 6713 -> 6460 (M = 2), 6725 -> 6120 (M = 4), 6108 -> 5346 (M = 3)
+    // and ADOPT N = 1 6447 -> 6248.  The 64-element chunks of M >= 5 keep
+    // the persistent grid (M = 8, ~350M workload: 6504 -> 6409).
     auto kernel = step_sync_kernel<BASE, N, GDT, CLIP, M>;
-    static const int per_sm = blocks_per_sm(kernel);
-    const int grid = persistent_grid(per_sm, num_sms, a.n_padded / FusedShape<M>::kChunk);
+    int grid;
+    if constexpr (FusedShape<M>::kChunk >= 128 && (N >= 2 || BASE == MTDAO_BASE_SGDM)) {
+        grid = stream_grid(a.n_padded / FusedShape<M>::kChunk);
+    } else {
+        static const int per_sm = blocks_per_sm(kernel);
+        grid = persistent_grid(per_sm, num_sms, a.n_padded / FusedShape<M>::kChunk);
+    }
     kernel<<<grid, kThreads, 0, stream>>>(a);
     return cudaGetLastError();
 }
