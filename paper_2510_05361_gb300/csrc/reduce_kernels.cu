@@ -67,11 +67,21 @@ __global__ void __launch_bounds__(kThreads) sync_kernel(const SyncArgs a) {
 
 template <int MT>
 cudaError_t launch_sync_t(const SyncArgs &a, int num_sms, cudaStream_t stream) {
-    static const int per_sm = blocks_per_sm(sync_kernel<MT>);
+    // M = 2, 4, 8 (replicas held in registers): one float4 position per
+    // thread, like the local step's stream_grid (flat 2^27, all states, GB/s
+    // against the persistent grid: M = 2 6342 -> 7098, M = 4 6447 -> 7025,
+    // M = 8 6546 -> 6941).  The streamed runtime-M loop keeps the persistent
+    // grid (M = 3: 6257, one position per thread 5591).
     const int64_t nv = a.n_padded / 4;
-    int64_t gx = static_cast<int64_t>(per_sm) * num_sms / (a.n_sel > 0 ? a.n_sel : 1);
     const int64_t need = (nv + kThreads - 1) / kThreads;
-    if (gx > need) gx = need;
+    int64_t gx;
+    if constexpr (MT > 0) {
+        gx = need > 0x7fffffff ? 0x7fffffff : need;
+    } else {
+        static const int per_sm = blocks_per_sm(sync_kernel<MT>);
+        gx = static_cast<int64_t>(per_sm) * num_sms / (a.n_sel > 0 ? a.n_sel : 1);
+        if (gx > need) gx = need;
+    }
     if (gx < 1) gx = 1;
     dim3 grid(static_cast<unsigned>(gx), static_cast<unsigned>(a.n_sel));
     sync_kernel<MT><<<grid, kThreads, 0, stream>>>(a);
