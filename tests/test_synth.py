@@ -64,3 +64,48 @@ def test_padding_is_zero():
         inside[off:off + num] = True
     assert np.all(g[~inside] == 0) and np.all(x[~inside] == 0)
     assert np.all(g[inside] != 0)
+
+
+def _rosenbrock(x):
+    a, b = x[0::2], x[1::2]
+    return float(np.sum((1.0 - a) ** 2 + 100.0 * (b - a * a) ** 2))
+
+
+def _central_diff(f, x, h=1e-6):
+    g = np.empty_like(x)
+    for i in range(x.size):
+        e = np.zeros_like(x)
+        e[i] = h
+        g[i] = (f(x + e) - f(x - e)) / (2 * h)
+    return g
+
+
+def test_toy_gradients_match_their_objectives():
+    """Without noise the toy gradients are the derivatives of the two
+    objectives (quadratic sum lam x^2 / 2 of Figure 2, Rosenbrock pairs of
+    Figure 1), checked against central differences of the objectives
+    themselves; the Rosenbrock minimum (1, 1) has zero gradient."""
+    rng = np.random.default_rng(7)
+    x = rng.uniform(-1.5, 1.5, size=(3, 12))
+    lam = rng.uniform(0.1, 10.0, size=12)
+    gq = G.toy_grad("quadratic", x, 1, 0, 0.0, lam=lam)
+    gr = G.toy_grad("rosenbrock", x, 1, 0, 0.0)
+    for m in range(3):
+        fq = lambda v: float(np.sum(lam * v * v) / 2)
+        np.testing.assert_allclose(gq[m], _central_diff(fq, x[m]), rtol=1e-6, atol=1e-6)
+        np.testing.assert_allclose(gr[m], _central_diff(_rosenbrock, x[m]), rtol=1e-6, atol=1e-4)
+    assert np.all(G.toy_grad("rosenbrock", np.ones((2, 6)), 1, 0, 0.0) == 0.0)
+
+
+def test_toy_gradient_noise():
+    """sigma scales standard normal noise that depends on the worker, the
+    step and the index, and not on x."""
+    x = np.zeros((2, 1 << 16))
+    g = G.toy_grad("quadratic", x, 5, 3, 0.5, lam=np.ones(1 << 16))
+    assert abs(g.mean()) < 0.01 and abs(g.std() - 0.5) < 0.01
+    assert not np.array_equal(g[0], g[1])
+    g_next = G.toy_grad("quadratic", x, 5, 4, 0.5, lam=np.ones(1 << 16))
+    assert not np.array_equal(g, g_next)
+    x2 = np.full((2, 1 << 16), 3.0)
+    g2 = G.toy_grad("quadratic", x2, 5, 3, 0.5, lam=np.ones(1 << 16))
+    np.testing.assert_allclose(g2 - 3.0, g, atol=1e-12)
