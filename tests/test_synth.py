@@ -1,5 +1,6 @@
 """The seeded input generators: determinism, distributions, padding."""
 import numpy as np
+import pytest
 
 from synth import generators as G
 from synth import workloads as W
@@ -109,3 +110,20 @@ def test_toy_gradient_noise():
     x2 = np.full((2, 1 << 16), 3.0)
     g2 = G.toy_grad("quadratic", x2, 5, 3, 0.5, lam=np.ones(1 << 16))
     np.testing.assert_allclose(g2 - 3.0, g, atol=1e-12)
+
+
+@pytest.mark.parametrize("name, d, ffn, blocks, total", [
+    ("gpt2_small", 768, 3072, 12, 123_570_432),
+    ("decoder_350m", 1024, 4096, 24, 353_553_408),
+    ("decoder_1b", 2048, 8192, 24, 1_311_086_592),
+])
+def test_decoder_lists_count_the_architecture(name, d, ffn, blocks, total):
+    """The named parameter lists hold V*d + L*(4 d^2 + 2 d F + 4 d) + 2 d
+    values (embedding; per block qkv, projection, two FFN matrices and two
+    layer norms; final layer norm) in 1 + 8 L + 2 tensors, all multiples of
+    8, so the padded layout adds nothing before the slab's last tail."""
+    shapes = W.WORKLOADS[name]["shapes"]
+    assert len(shapes) == 1 + 8 * blocks + 2
+    assert sum(shapes) == W.VOCAB * d + blocks * (4 * d * d + 2 * d * ffn + 4 * d) + 2 * d == total
+    assert all(s % 8 == 0 for s in shapes)
+    assert W.layout(shapes)["n_padded"] == -(-total // 256) * 256
