@@ -91,3 +91,25 @@ def test_reference_arm_json_line():
     e = d["e2e"]
     assert e["value"] == d["value"] and e["unit"] == d["unit"]
     assert e["h2d_bytes_per_step"] == 0 and e["d2h_bytes_per_step"] == 0
+
+
+def test_step_kernel_traffic_gate(tmp_path, monkeypatch):
+    """bench.py reports the committed DRAM traffic only for the kernel
+    instance and the kernel source it was captured from, scaled by the
+    elements of the launch it times."""
+    sys.path.insert(0, ROOT)
+    import bench
+    name = bench.step_kernel_name({"base": "adam", "n_mom": 3, "clip_mode": "none"}, "f32")
+    assert name == "step_kernel<0, 3, 0, 0>"
+    assert bench.step_kernel_name({"base": "adopt", "n_mom": 2}, "bf16") == "step_kernel<1, 2, 1, 0>"
+    rec = tmp_path / "traffic.txt"
+    rec.write_text("# capture\nkernel=%s\nelements=1000\ndram_bytes=44000\nsource_sha=%s\n"
+                   % (name, bench.source_sha()))
+    monkeypatch.setattr(bench, "TRAFFIC_FILE", str(rec))
+    assert bench.measured_traffic(name, 5000) == 220000
+    assert bench.measured_traffic("step_kernel<1, 2, 1, 0>", 5000) is None
+    rec.write_text("kernel=%s\nelements=1000\ndram_bytes=44000\nsource_sha=0000000000000000\n" % name)
+    assert bench.measured_traffic(name, 5000) is None
+    monkeypatch.setattr(bench, "TRAFFIC_FILE", str(tmp_path / "missing.txt"))
+    assert bench.measured_traffic(name, 5000) is None
+
