@@ -8,6 +8,7 @@ counts every rank's units, and the reference arm runs on rank 0 only.
 import json
 import os
 import socket
+import statistics
 import subprocess
 import sys
 
@@ -113,3 +114,22 @@ def test_step_kernel_traffic_gate(tmp_path, monkeypatch):
     monkeypatch.setattr(bench, "TRAFFIC_FILE", str(tmp_path / "missing.txt"))
     assert bench.measured_traffic(name, 5000) is None
 
+
+
+def test_clock_sample_summary():
+    """The clocks record of the bench line: median SM clock under load,
+    maximum clock, slowdown reasons seen active; idle and malformed samples
+    do not count."""
+    sys.path.insert(0, ROOT)
+    import bench
+    idle = "0, 1965, 2070, 180.5, 0x0000000000000001, Not Active, Not Active, Not Active, Not Active"
+    busy = "0, 2070, 2070, 950.0, 0x0000000000000000, Not Active, Not Active, Not Active, Not Active"
+    capped = "0, 1890, 2070, 1390.2, 0x0000000000000004, Not Active, Not Active, Not Active, Active"
+    slow = "0, 1500, 2070, 900.0, 0x0000000000000008, Active, Not Active, Not Active, Not Active"
+    s = bench.parse_clock_samples([idle, busy, busy, "garbage", "0, [N/A], 2070, 1, x, a, b, c, d"])
+    assert s["sm_mhz"] == 2070.0 and s["sm_max_mhz"] == 2070.0 and s["reasons"] == []
+    assert s["samples"] == 3 and s["power_w_max"] == 950.0
+    s = bench.parse_clock_samples([busy, capped, capped, slow])
+    assert s["reasons"] == ["hw_slowdown", "sw_power_cap"]
+    assert s["sm_mhz"] == statistics.median([2070.0, 1890.0, 1890.0, 1500.0])
+    assert bench.parse_clock_samples([])["reasons"] == ["no samples"]
