@@ -53,7 +53,8 @@ typedef enum {
     MTDAO_ERR_INVALID = -1,      /* bad argument or configuration */
     MTDAO_ERR_OOM = -2,          /* device or pinned-host allocation failed */
     MTDAO_ERR_CUDA = -3,         /* a CUDA runtime call or launch failed */
-    MTDAO_ERR_ALIGN = -4,        /* a pointer is not 16-byte aligned */
+    MTDAO_ERR_ALIGN = -4,        /* a pointer is not aligned as the call requires (16 bytes
+                                    for vectors, 8 bytes for double outputs) */
     MTDAO_ERR_STATE = -5         /* call not allowed in the handle's state */
 } mtdao_status;
 
@@ -196,7 +197,12 @@ int mtdao_comm_reduction(const mtdao_config *cfg, double *factor_out);
 
 /*
  * Create a handle on the current CUDA device for M replicas of the tensor
- * list tensor_numel[0..n_tensors-1] (host array).  Allocates the state
+ * list tensor_numel[0..n_tensors-1] (host array).  This takes the inputs of
+ * the "Require" lists of Algorithms 1-3: the number of workers M, the
+ * hyper-parameters in *cfg (decay rates beta_j and beta_2, weights omega_j,
+ * epsilon, the sync periods K_x, K_j, K_v, the clipping rule) and the shape
+ * of the parameters x (the learning rates eta_t arrive per step, the
+ * initial x_0 through mtdao_set_params).  Allocates the state
  * arena (num_states * M * n_padded fp32) and workspaces, zeroes every state
  * and sets the step counter t to 0.  cuda_stream is a cudaStream_t (NULL =
  * legacy default stream).  On failure *out is NULL and the reason is
@@ -241,6 +247,9 @@ int mtdao_set_params(mtdao_handle h, const float *x0_dev);
  *   2 <= M <= 8 and M = 16; other M fall back to a separate averaging
  *   pass.
  * With MTDAO_CLIP_GLOBAL_NORM a reduction pass over grads precedes the step.
+ * With adopt_prev_v (the original ADOPT order) step 0 runs a separate pass
+ * that writes v = g_0^2 and reads or writes nothing else, so u and x keep
+ * their initial values even where g_0 is not finite.
  * Errors: MTDAO_ERR_INVALID (dtype, mask bits beyond the states),
  * MTDAO_ERR_ALIGN, MTDAO_ERR_CUDA.  On error t is unchanged.
  */
@@ -290,7 +299,8 @@ int mtdao_sync(mtdao_handle h, uint32_t mask);
  * mtdao_sync plus the paper's cross-worker diagnostics (section 4.1, "Other
  * Metrics"), formed in the same pass over the replicas at no extra state
  * traffic.  For every state s in mask, in increasing state order, stats_dev
- * (device, caller-owned, popcount(mask) * (2 + 2M) doubles) receives, from
+ * (device, caller-owned, 8-byte aligned, popcount(mask) * (2 + 2M) doubles)
+ * receives, from
  * the replicas before they are averaged and their fp32 mean s_bar:
  *   [0]              (1/M) sum_m ||s_m - s_bar||^2   cross-worker variance
  *   [1]              ||s_bar||^2
@@ -324,7 +334,7 @@ int mtdao_track_anchor(mtdao_handle h, uint32_t state_mask);
 /*
  * Change diagnostics of one state against its anchor a, read-only (no state
  * changes), fixed-order sums.  With s_bar the replica mean an average would
- * store now, out_dev (device, 2M + 2 doubles) gets
+ * store now, out_dev (device, 8-byte aligned, 2M + 2 doubles) gets
  *   [m]        ||s_m - a||^2                 m = 0..M-1  (local change, for x
  *                                                          the pseudo-gradient)
  *   [M + m]    <s_m - a, s_bar - a>
@@ -344,9 +354,13 @@ int mtdao_sync_due(mtdao_handle h, uint32_t *mask_out);
 /*
  * Squared L2 norm of each replica's flattened gradient (the quantity that
  * clip(g, rho) of Algorithms 1 and 3 is based on): out_dev (device, M
- * doubles, caller-owned) receives sum_i g[m][i]^2.  Deterministic: fixed
- * grid and fixed reduction order.  Uses a handle-owned workspace of partial
- * sums.
+ * doubles, caller-owned, 8-byte aligned) receives sum_i g[m][i]^2.
+ * Deterministic: fixed grid and fixed reduction order.  Squares are summed
+ * in fp32 with compensation where they stay within fp32's range; groups of
+ * four values whose squares overflow or underflow fp32 (|g| above ~1e19 or
+ * below ~1e-19) are summed in fp64, so every finite gradient gives a finite,
+ * accurate sum.  Uses a handle-owned workspace of partial sums.
+ * Errors: MTDAO_ERR_INVALID, MTDAO_ERR_ALIGN, MTDAO_ERR_CUDA.
  */
 int mtdao_grad_sqnorm(mtdao_handle h, const void *grads_dev, int32_t grad_dtype,
                       double *out_dev);
@@ -355,7 +369,7 @@ int mtdao_grad_sqnorm(mtdao_handle h, const void *grads_dev, int32_t grad_dtype,
  * Gradient health check (the paper has no counterpart; NaN and Inf
  * gradients otherwise propagate into every state of the replica, as the
  * algorithms written out would propagate them): out_dev (device, M doubles,
- * caller-owned) receives the number of NaN or +-Inf values in replica m's
+ * caller-owned, 8-byte aligned) receives the number of NaN or +-Inf values in replica m's
  * gradient, exact.  A caller can skip a step whose count is nonzero (e.g.
  * an overflow of bf16 gradients).  Same grid, workspace and
  * determinism as mtdao_grad_sqnorm; reads the gradient once (g_b bytes per
@@ -381,19 +395,24 @@ int mtdao_grad_nonfinite(mtdao_handle h, const void *grads_dev, int32_t grad_dty
  * loads the library holds until the process exits.  A call needs
  * M * blocks_per_replica slots (blocks_per_replica = max(1, 4 * SMs / M),
  * the grid of mtdao_grad_sqnorm, so both return the same bits); a call that
- * would need more fails with MTDAO_ERR_INVALID and a message.  Every slot a
+ * would need more fails with MTDAO_ERR_INVALID and a message.  On a 152-SM
+ * GB300 a call needs at most max(M, 608) <= 1024 slots, so every valid M
+ * fits; the limit binds only on devices with more than 1024 SMs.  Every slot a
  * call reads is written earlier in the same call, so nothing has to be
  * cleared between calls; the array keeps the last call's partial sums.
  * All calls on a device share the array: calls whose GPU work overlaps (on
  * different streams or from different threads) race and return garbage.
  *
  * Set-up: the first call on a device (with that device current) looks up
- * the array's device address with cudaGetSymbolAddress and caches it; make
- * that first call before any stream capture begins.
+ * the array's device address with cudaGetSymbolAddress and caches it, keyed
+ * by the device and the unique id of its current context; the first call
+ * after the context changed (after a cudaDeviceReset, say) looks it up
+ * again.  Make the first call on a device before any stream capture begins.
  *
  * grads_dev: device, [M][n_padded] of grad_dtype, 16-byte aligned;
  * n_padded a positive multiple of 256; 1 <= M <= MTDAO_MAX_REPLICAS.
- * out_dev: device, M doubles (caller-owned), receives sum_i g[m][i]^2.
+ * out_dev: device, M doubles (caller-owned, 8-byte aligned), receives
+ *   sum_i g[m][i]^2 (computed as by mtdao_grad_sqnorm).
  * cuda_stream: cudaStream_t the work is enqueued on (asynchronous).
  * Errors: MTDAO_ERR_INVALID, MTDAO_ERR_ALIGN, MTDAO_ERR_CUDA; the message is
  * available from mtdao_last_error(NULL) in the calling thread.
@@ -404,7 +423,13 @@ int mtdao_grad_sqnorm_static(const void *grads_dev, int32_t grad_dtype, int32_t 
 
 /* ------------------------------------------------------------------ state access */
 
-/* Device pointer to state `state` of replica `replica` ([n_padded] fp32). */
+/*
+ * Device pointer to state `state` of replica `replica` ([n_padded] fp32,
+ * owned by the handle, valid until destroy): the outputs of Algorithms 1-3
+ * ("Ensure x_T, {u^j}, v") are read here, x = state 0 of any replica after
+ * an average of x, u^j = state j, v = state N+1.  Errors: MTDAO_ERR_INVALID
+ * for a state or replica out of range or a NULL dev_ptr.
+ */
 int mtdao_get_state_ptr(mtdao_handle h, int32_t state, int32_t replica, float **dev_ptr);
 
 /* Copy one state vector to host memory ([n_padded] floats); synchronises. */
@@ -417,7 +442,10 @@ int mtdao_copy_state_from_host(mtdao_handle h, int32_t state, int32_t replica,
 /*
  * Layout of the handle: *n_padded, *n_tensors, *M, *n_states and a pointer
  * to the handle-owned offsets array (valid until destroy).  Any output
- * pointer may be NULL.
+ * pointer may be NULL.  This maps the flattened state vectors back to the
+ * caller's tensors, the shape in which Algorithms 1-3 hand back their
+ * outputs x_T, {u^j}, v ("Ensure"): tensor k of state s, replica m starts at
+ * state pointer + offset_k.  Host-only, no device access.
  */
 int mtdao_layout(mtdao_handle h, int64_t *n_padded, int32_t *n_tensors, int32_t *M,
                  int32_t *n_states, const int64_t **tensor_offsets);

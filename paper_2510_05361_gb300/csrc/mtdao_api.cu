@@ -227,12 +227,6 @@ StepScalars step_scalars(const mtdao_config *c, int64_t t, double lr) {
                    ? static_cast<float>(std::pow(static_cast<double>(k), 0.25))
                    : INFINITY;
     s.prev_v = prev_v ? 1 : 0;
-    if (prev_v && t == 0) {
-        // original ADOPT order, step 0: v = g_0^2 and nothing else moves
-        s.c2 = 1.0f;
-        for (int j = 0; j < c->n_mom; ++j) s.c1[j] = 0.0f;
-        s.neg_lr = 0.0f;
-    }
     return s;
 }
 
@@ -278,6 +272,7 @@ int check_handle(mtdao_ctx *h) {
 }
 
 bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+bool aligned8(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 7u) == 0; }
 
 int select_device(mtdao_ctx *h) {
     int cur = -1;
@@ -567,6 +562,20 @@ extern "C" int mtdao_step(mtdao_handle h, const void *grads_dev, int32_t grad_dt
     if (int rc = select_device(h)) return rc;
 
     const mtdao_config *c = &h->cfg;
+    const uint32_t avg_mask = h->M > 1 ? sync_mask : 0u;
+    if (c->base == MTDAO_BASE_ADOPT && c->adopt_prev_v && h->step == 0) {
+        // Original ADOPT order, step 0: v = g_0^2 on every replica and
+        // nothing else moves; then the averages due at the end of the step.
+        float *v = h->arena + static_cast<int64_t>(1 + c->n_mom) * h->M * h->n_padded;
+        cudaError_t e = launch_adopt_init_v(v, grads_dev, grad_dtype, static_cast<int64_t>(h->M) * h->n_padded,
+                                            h->stream);
+        if (e != cudaSuccess) return cuda_fail(h, e, "ADOPT initial second-moment launch");
+        if (avg_mask != 0)
+            if (int rc = enqueue_sync(h, avg_mask)) return rc;
+        if (int rc = refresh_anchor(h, sync_mask)) return rc;
+        ++h->step;
+        return MTDAO_OK;
+    }
     const bool clip = c->clip_mode == MTDAO_CLIP_GLOBAL_NORM;
     if (clip) {
         cudaError_t e = launch_grad_sqnorm(grads_dev, grad_dtype, h->M, h->n_padded, h->norm_blocks,
@@ -582,7 +591,7 @@ extern "C" int mtdao_step(mtdao_handle h, const void *grads_dev, int32_t grad_dt
     a.n_padded = h->n_padded;
     a.stride = static_cast<int64_t>(h->M) * h->n_padded;
     a.M = h->M;
-    a.sync_mask = h->M > 1 ? sync_mask : 0u;
+    a.sync_mask = avg_mask;
     a.sc = step_scalars(c, h->step, lr);
 
     cudaError_t e;
@@ -686,6 +695,7 @@ extern "C" int mtdao_sync_stats(mtdao_handle h, uint32_t mask, double *stats_dev
     Range range("mtdao_sync_stats");
     if (int rc = check_handle(h)) return rc;
     if (stats_dev == nullptr) return set_error(h, MTDAO_ERR_INVALID, "stats is NULL");
+    if (!aligned8(stats_dev)) return set_error(h, MTDAO_ERR_ALIGN, "stats not 8-byte aligned");
     if (mask >> h->n_states) return set_error(h, MTDAO_ERR_INVALID, "sync mask 0x%x has bits beyond "
                                               "the %d states", mask, h->n_states);
     if (mask == 0) return MTDAO_OK;
@@ -742,6 +752,7 @@ extern "C" int mtdao_pseudo_grad_stats(mtdao_handle h, int32_t state, double *ou
     Range range("mtdao_pseudo_grad_stats");
     if (int rc = check_handle(h)) return rc;
     if (out_dev == nullptr) return set_error(h, MTDAO_ERR_INVALID, "out is NULL");
+    if (!aligned8(out_dev)) return set_error(h, MTDAO_ERR_ALIGN, "out not 8-byte aligned");
     if (state < 0 || state >= h->n_states) return set_error(h, MTDAO_ERR_INVALID, "state %d out of range", state);
     if (h->anchor[state] == nullptr)
         return set_error(h, MTDAO_ERR_STATE, "state %d has no anchor: track it with mtdao_track_anchor", state);
@@ -772,6 +783,7 @@ extern "C" int mtdao_grad_nonfinite(mtdao_handle h, const void *grads_dev, int32
     if (grads_dev == nullptr || out_dev == nullptr)
         return set_error(h, MTDAO_ERR_INVALID, "grads or out is NULL");
     if (!aligned16(grads_dev)) return set_error(h, MTDAO_ERR_ALIGN, "grads not 16-byte aligned");
+    if (!aligned8(out_dev)) return set_error(h, MTDAO_ERR_ALIGN, "out not 8-byte aligned");
     if (grad_dtype != MTDAO_F32 && grad_dtype != MTDAO_BF16)
         return set_error(h, MTDAO_ERR_INVALID, "unknown gradient dtype %d", grad_dtype);
     if (int rc = select_device(h)) return rc;
@@ -788,6 +800,7 @@ extern "C" int mtdao_grad_sqnorm(mtdao_handle h, const void *grads_dev, int32_t 
     if (grads_dev == nullptr || out_dev == nullptr)
         return set_error(h, MTDAO_ERR_INVALID, "grads or out is NULL");
     if (!aligned16(grads_dev)) return set_error(h, MTDAO_ERR_ALIGN, "grads not 16-byte aligned");
+    if (!aligned8(out_dev)) return set_error(h, MTDAO_ERR_ALIGN, "out not 8-byte aligned");
     if (grad_dtype != MTDAO_F32 && grad_dtype != MTDAO_BF16)
         return set_error(h, MTDAO_ERR_INVALID, "unknown gradient dtype %d", grad_dtype);
     if (int rc = select_device(h)) return rc;

@@ -33,7 +33,8 @@ struct StepScalars {
     float sv;                        // Adam: 1 / sqrt(1 - beta_2^(t+1)), or 1
     float eps;                       // epsilon
     float clip_c;                    // ADOPT clamp bound c_t (+inf when not clipping)
-    int prev_v;                      // ADOPT: normalise with the previous v (original order)
+    int prev_v;                      // ADOPT: normalise with the previous v (original order);
+                                     // its step 0 runs launch_adopt_init_v instead
 };
 
 struct StepArgs {
@@ -65,6 +66,11 @@ cudaError_t launch_step(int base, int n_mom, int grad_dtype, bool clip, const St
 // otherwise (the caller then runs launch_step followed by launch_sync).
 cudaError_t launch_step_sync(int base, int n_mom, int grad_dtype, bool clip, const StepArgs &a,
                              int num_sms, cudaStream_t stream);
+
+// Step 0 of the original ADOPT order: v = g^2 over count elements (all
+// replicas' v slabs, contiguous), nothing else touched.
+cudaError_t launch_adopt_init_v(float *v, const void *grads, int grad_dtype, int64_t count,
+                                cudaStream_t stream);
 
 // Replace each selected state by its mean over the M replicas.
 cudaError_t launch_sync(const SyncArgs &a, int num_sms, cudaStream_t stream);

@@ -10,6 +10,7 @@
 // buffer and has no handle.  mtdao_grad_sqnorm_static serves them: its
 // scratch (the per-block partial sums) is a fixed file-scope device array
 // that exists for as long as the library is loaded on a device.
+#include <cuda.h>
 #include <cuda_runtime.h>
 
 #include <cstdio>
@@ -28,16 +29,57 @@ static __device__ __align__(256) double g_sqnorm_scratch[MTDAO_STATIC_SCRATCH_DO
 
 constexpr int kMaxDevices = 64;
 std::mutex g_setup_mutex;
-void *g_scratch_addr[kMaxDevices] = {};
+
+// Per device: the array's device address and the unique id of the context
+// it was looked up in.  A device reset (cudaDeviceReset) destroys the
+// primary context and a later call runs in a new one, where the module is
+// loaded again and the array may sit elsewhere; the id tells the two apart
+// (context ids are never reused within a process).
+struct ScratchAddr {
+    void *ptr = nullptr;
+    unsigned long long ctx_id = 0;
+};
+ScratchAddr g_scratch[kMaxDevices];
+
+// cuCtxGetId from the driver, found once through the runtime (so the
+// library needs no link-time dependency on libcuda).  nullptr if the
+// driver does not offer it; the cache is then kept per device only.
+using CtxGetIdFn = CUresult (*)(CUcontext, unsigned long long *);
+CtxGetIdFn ctx_get_id() {
+    static CtxGetIdFn fn = [] {
+        void *p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuCtxGetId", &p, 12000, cudaEnableDefault, &q) != cudaSuccess ||
+            q != cudaDriverEntryPointSuccess) {
+            cudaGetLastError();
+            p = nullptr;
+        }
+        return reinterpret_cast<CtxGetIdFn>(p);
+    }();
+    return fn;
+}
+
+// Id of the context current on this thread, or 0 if there is none yet (a
+// thread whose first runtime call this is) or it cannot be told.
+unsigned long long current_ctx_id() {
+    CtxGetIdFn fn = ctx_get_id();
+    unsigned long long id = 0;
+    if (fn == nullptr || fn(nullptr, &id) != CUDA_SUCCESS) return 0;
+    return id;
+}
 
 // Device address of g_sqnorm_scratch on the current device.  In host code
 // the array's name is only a host-side stand-in, so the address is looked up
-// once per device (the first call on a device does this) and cached.
+// with cudaGetSymbolAddress (the first call on a device, and the first call
+// after its context changed, does this; the lookup also makes the device's
+// primary context current on this thread) and cached.
 int scratch_on_current_device(int dev, void **out) {
     if (dev < 0 || dev >= kMaxDevices)
         return mtdao::set_thread_error(MTDAO_ERR_INVALID, "device index beyond the supported 64");
     std::lock_guard<std::mutex> lock(g_setup_mutex);
-    if (g_scratch_addr[dev] == nullptr) {
+    ScratchAddr &slot = g_scratch[dev];
+    const unsigned long long id = current_ctx_id();
+    if (slot.ptr == nullptr || (id != 0 && id != slot.ctx_id)) {
         void *p = nullptr;
         const cudaError_t e = cudaGetSymbolAddress(&p, g_sqnorm_scratch);
         if (e != cudaSuccess || p == nullptr) {
@@ -46,9 +88,10 @@ int scratch_on_current_device(int dev, void **out) {
                      cudaGetErrorString(e));
             return mtdao::set_thread_error(MTDAO_ERR_CUDA, msg);
         }
-        g_scratch_addr[dev] = p;
+        slot.ptr = p;
+        slot.ctx_id = current_ctx_id();
     }
-    *out = g_scratch_addr[dev];
+    *out = slot.ptr;
     return MTDAO_OK;
 }
 
@@ -60,6 +103,8 @@ extern "C" int mtdao_grad_sqnorm_static(const void *grads_dev, int32_t grad_dtyp
         return mtdao::set_thread_error(MTDAO_ERR_INVALID, "grads or out is NULL");
     if ((reinterpret_cast<uintptr_t>(grads_dev) & 15u) != 0)
         return mtdao::set_thread_error(MTDAO_ERR_ALIGN, "grads not 16-byte aligned");
+    if ((reinterpret_cast<uintptr_t>(out_dev) & 7u) != 0)
+        return mtdao::set_thread_error(MTDAO_ERR_ALIGN, "out not 8-byte aligned");
     if (grad_dtype != MTDAO_F32 && grad_dtype != MTDAO_BF16)
         return mtdao::set_thread_error(MTDAO_ERR_INVALID, "unknown gradient dtype");
     if (M < 1 || M > MTDAO_MAX_REPLICAS)

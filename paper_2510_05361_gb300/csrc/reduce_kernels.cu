@@ -137,6 +137,18 @@ __device__ __forceinline__ float4 widen(GradWords<GDT> w) {
                            __uint_as_float(w.y << 16), __uint_as_float(w.y & 0xffff0000u));
 }
 
+// fp32 range of a position's sum of four squares that the Kahan sum takes:
+// above kSqHi a square or the sum may overflow (|g| above ~1.8e19 squares to
+// Inf in fp32), below kSqLo a square may have lost bits to underflow (|g|
+// below ~1e-19).  Positions outside it (and NaN / Inf) are summed in fp64
+// instead, where every finite fp32 value squares exactly enough; the all-zero
+// positions of padding and unused rows stay on the fp32 path.  A replica has
+// at least 256 threads and, to fit in device memory, fewer than 2^34
+// elements, so a thread adds fewer than 2^24 positions of at most 2^100:
+// the fp32 sum stays finite.
+constexpr float kSqHi = 0x1p100f;
+constexpr float kSqLo = 0x1p-100f;
+
 template <int GDT>
 __global__ void __launch_bounds__(kNormThreads, 4) sqnorm_partial_kernel(const void *g, int64_t n,
                                                                       double *partial) {
@@ -145,6 +157,7 @@ __global__ void __launch_bounds__(kNormThreads, 4) sqnorm_partial_kernel(const v
     const int64_t nv = n / 4;
     const int64_t T = static_cast<int64_t>(nb) * blockDim.x;
     float sum = 0.0f, comp = 0.0f;
+    double wide = 0.0;                 // positions outside [kSqLo, kSqHi]
     for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < nv;
          i += kNormUnroll<GDT> * T) {
         GradWords<GDT> w[kNormUnroll<GDT>];
@@ -155,13 +168,21 @@ __global__ void __launch_bounds__(kNormThreads, 4) sqnorm_partial_kernel(const v
         for (int u = 0; u < kNormUnroll<GDT>; ++u) {
             if (i + u * T >= nv) break;
             const float4 q = widen<GDT>(w[u]);
-            const float y = fmaf(q.x, q.x, fmaf(q.y, q.y, fmaf(q.z, q.z, __fmul_rn(q.w, q.w)))) - comp;
+            const float p = fmaf(q.x, q.x, fmaf(q.y, q.y, fmaf(q.z, q.z, __fmul_rn(q.w, q.w))));
+            const bool tiny = p < kSqLo && ((__float_as_uint(q.x) | __float_as_uint(q.y) | __float_as_uint(q.z) |
+                                             __float_as_uint(q.w)) & 0x7fffffffu) != 0u;
+            if (!(p <= kSqHi) || tiny) {
+                const double a = q.x, b = q.y, c = q.z, d = q.w;
+                wide += fma(a, a, fma(b, b, fma(c, c, d * d)));
+                continue;
+            }
+            const float y = p - comp;
             const float t = sum + y;
             comp = (t - sum) - y;
             sum = t;
         }
     }
-    const double total = block_sum(static_cast<double>(sum) - static_cast<double>(comp));
+    const double total = block_sum((static_cast<double>(sum) - static_cast<double>(comp)) + wide);
     if (threadIdx.x == 0) partial[static_cast<int64_t>(m) * nb + blockIdx.x] = total;
 }
 

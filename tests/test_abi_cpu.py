@@ -185,3 +185,24 @@ def test_binding_gradient_dtype_code(P):
         code(torch.zeros(3), P.BF16)
     with pytest.raises(ValueError):
         code(torch.zeros(3, dtype=torch.bfloat16), P.F32)
+
+
+def test_static_norm_checks_arguments_before_touching_a_device(P):
+    """mtdao_grad_sqnorm_static rejects NULL, misaligned or out-of-range
+    arguments before it makes any CUDA call (the pointers below are never
+    dereferenced), with the code the header states."""
+    g, out = 0x10000, 0x20000          # 16-byte aligned stand-ins, never read
+    cases = [((0, P.F32, 2, 256, out), P.ERR_INVALID),
+             ((g, P.F32, 2, 256, 0), P.ERR_INVALID),
+             ((g + 8, P.F32, 2, 256, out), P.ERR_ALIGN),
+             ((g, P.F32, 2, 256, out + 4), P.ERR_ALIGN),
+             ((g, 7, 2, 256, out), P.ERR_INVALID),
+             ((g, P.F32, 0, 256, out), P.ERR_INVALID),
+             ((g, P.F32, P.MAX_REPLICAS + 1, 256, out), P.ERR_INVALID),
+             ((g, P.BF16, 2, 100, out), P.ERR_INVALID),
+             ((g, P.BF16, 2, 0, out), P.ERR_INVALID)]
+    for args, code in cases:
+        with pytest.raises(P.MTDAOError) as e:
+            P.mtdao_grad_sqnorm_static(*args, 0)
+        assert e.value.code == code, (args, e.value)
+        assert P.mtdao_last_error(None)

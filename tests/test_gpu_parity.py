@@ -143,6 +143,72 @@ def test_grad_sqnorm(P, gdt):
 
 
 @pytest.mark.parametrize("gdt", ["f32", "bf16"])
+def test_grad_sqnorm_extreme_range(P, gdt):
+    """Sums of squares whose terms leave fp32's range: replica 0 holds a few
+    finite values whose squares overflow fp32 (1.5e19 squares to 2.25e38,
+    four of them to more than the largest float; 3e30 and -1e38 overflow
+    outright), replica 1 is scaled to ~1e-25 (every square underflows
+    fp32), replica 2 is ordinary.  Each must match the fp64 sum within
+    1e-6 relative, as the oracle's norm (fp64) does."""
+    M = 3
+    w = workload_dict([70000, 3, 1000], M, sigma=0.5, gdt=gdt)
+    lay = W.layout(w["shapes"])
+    g = host_grads(w, lay, SEED_G, 0, np.arange(lay["n_padded"]))
+    g[0, [4, 5, 6, 7]] = np.float32(1.5e19)
+    g[0, 100] = np.float32(-1.5e19)
+    g[0, 2000] = np.float32(3e30)
+    g[0, 3001] = np.float32(-1e38)
+    g[1] *= np.float32(2e-25)
+    if gdt == "bf16":
+        g = G.round_bf16(g)
+    assert np.all(np.isfinite(g))
+    eng = P.MTDAO(w["opt"], M, w["shapes"])
+    out = torch.zeros(M, dtype=torch.float64, device="cuda")
+    gd = to_dev(g, gdt)
+    P.mtdao_grad_sqnorm(eng.h, gd.data_ptr(), P.BF16 if gdt == "bf16" else P.F32, out.data_ptr())
+    got = out.cpu().numpy()
+    expect = np.sum(g.astype(np.float64) ** 2, axis=1)
+    assert np.all(np.isfinite(got)), got
+    assert np.max(np.abs(got - expect) / expect) < 1e-6, (got, expect)
+    eng.close()
+
+
+@pytest.mark.parametrize("gdt", ["f32", "bf16"])
+@pytest.mark.parametrize("base", ["adam", "sgdm"])
+def test_global_norm_clip_parity_with_huge_gradients(P, base, gdt):
+    """clip(g, rho) when a replica's gradient holds finite values whose fp32
+    squares overflow a four-term sum (1.5e19 each): the norm is formed in
+    range, the clip factor is the oracle's tiny one rather than 0, and every
+    state matches the oracle (the states themselves stay within fp32)."""
+    M = 4
+    w = workload_dict([5000, 3001, 17], M, base=base, betas=(0.9, 0.999), clip="global_norm",
+                      rho=1.0, px=3, pu=2, pv=3, sigma=1.0, gdt=gdt)
+    lay = W.layout(w["shapes"])
+    n = lay["n_padded"]
+    idx = np.arange(n)
+    lr = w["opt"]["lr"]
+    eng = P.MTDAO(w["opt"], M, w["shapes"])
+    x0 = G.init_params(w, lay, SEED_I, idx)
+    eng.set_params(torch.from_numpy(x0).cuda())
+    from oracle.oracle import Oracle
+    o = Oracle(w["opt"], M, n, x0=x0.astype(np.float64))
+    T = 6
+    for t in range(T):
+        g = host_grads(w, lay, SEED_G, t, idx)
+        if t in (1, 4):
+            g[1, 8:12] = np.float32(1.5e19)
+            g[2, 5003] = np.float32(-1.5e19)
+            if gdt == "bf16":
+                g = G.round_bf16(g)             # what the device sees after its bf16 rounding
+        eng.step(to_dev(g, gdt), lr, eng.sync_due())
+        o.step(t, lr, g.astype(np.float64))
+    o.settle(T)
+    torch.cuda.synchronize()
+    compare(gpu_states(eng, w["opt"]), o.states())
+    eng.close()
+
+
+@pytest.mark.parametrize("gdt", ["f32", "bf16"])
 def test_grad_nonfinite_counts(P, gdt):
     """mtdao_grad_nonfinite counts exactly the NaN / +-Inf values planted in
     each replica's gradient (counts known by construction); the largest
@@ -316,23 +382,99 @@ def test_checkpoint_resume_is_bitwise_equal(P):
     resumed.close()
 
 
-def test_nonfinite_gradients_propagate_like_the_oracle(P):
-    w = workload_dict([1000], 2, betas=(0.9,), px=0, pu=0, pv=0)
+NONFINITE_VARIANTS = {
+    "adam": dict(base="adam"),
+    "adam_clip": dict(base="adam", clip="global_norm", rho=1.0),
+    "adopt": dict(base="adopt", beta2=0.9999),
+    "adopt_prev_v": dict(base="adopt", beta2=0.9999, clip="elementwise"),
+    "sgdm": dict(base="sgdm"),
+}
+
+
+@pytest.mark.parametrize("t_plant", [0, 2])
+@pytest.mark.parametrize("sync", ["plain", "fused_every2", "fused_every1"])
+@pytest.mark.parametrize("gdt", ["f32", "bf16"])
+@pytest.mark.parametrize("variant", sorted(NONFINITE_VARIANTS))
+def test_nonfinite_gradients_propagate_like_the_oracle(P, variant, gdt, sync, t_plant):
+    """NaN, +Inf and -Inf gradients planted in three of four replicas at
+    step 0 or 2, with no average, the fused average every second step, or
+    every step: the NaN/Inf positions of every state equal the oracle's and
+    the finite values agree within the tolerance.  The original ADOPT order
+    (step 0 only sets v = g_0^2, Algorithm 2 read as the original method)
+    must leave u and x finite when step 0's gradient is not."""
+    M = 4
+    period = {"plain": 0, "fused_every2": 2, "fused_every1": 1}[sync]
+    kw = dict(NONFINITE_VARIANTS[variant])
+    w = workload_dict([1000, 37], M, betas=(0.9, 0.99), px=period, pu=period, pv=period, gdt=gdt,
+                      lr=2.0 ** -8 if kw["base"] == "adopt" else 1e-3, **kw)
+    if variant == "adopt_prev_v":
+        w["opt"]["adopt_prev_v"] = True
     lay = W.layout(w["shapes"])
-    idx = np.arange(lay["n_padded"])
-    eng = P.MTDAO(w["opt"], 2, w["shapes"])
+    n = lay["n_padded"]
+    idx = np.arange(n)
+    lr = w["opt"]["lr"]
+    eng = P.MTDAO(w["opt"], M, w["shapes"])
     x0 = G.init_params(w, lay, SEED_I, idx)
     eng.set_params(torch.from_numpy(x0).cuda())
-    g = host_grads(w, lay, SEED_G, 0, idx)
-    g[0, 5] = np.nan
-    g[1, 9] = np.inf
-    eng.step(torch.from_numpy(g).cuda(), 1e-3, 0)
-    torch.cuda.synchronize()
     from oracle.oracle import Oracle
-    o = Oracle(w["opt"], 2, lay["n_padded"], x0=x0.astype(np.float64))
-    o.step(0, 1e-3, g.astype(np.float64))
-    compare(gpu_states(eng, w["opt"]), o.states())
+    o = Oracle(w["opt"], M, n, x0=x0.astype(np.float64))
+    T = 4
+    for t in range(T):
+        g = host_grads(w, lay, SEED_G, t, idx)
+        if t == t_plant:
+            g[0, 5] = np.nan
+            g[1, 9] = np.inf
+            g[2, lay["offsets"][1] + 3] = -np.inf
+        eng.step(to_dev(g, gdt), lr, eng.sync_due())
+        o.step(t, lr, g.astype(np.float64))
+    o.settle(T)
+    torch.cuda.synchronize()
+    got, ref = gpu_states(eng, w["opt"]), o.states()
+    compare(got, ref)                    # includes: non-finite positions are equal
+    if sync == "plain":
+        # no average: NaN and each sign of Inf where the oracle has them (after
+        # an average the compensated mean turns an infinite replica value into
+        # NaN, where an fp64 mean keeps the infinity; still non-finite)
+        for k in ref:
+            assert np.array_equal(np.isnan(got[k]), np.isnan(ref[k])), k
+            assert np.array_equal(np.isposinf(got[k]), np.isposinf(ref[k])), k
+            assert np.array_equal(np.isneginf(got[k]), np.isneginf(ref[k])), k
     eng.close()
+
+
+def test_original_adopt_step0_moves_nothing_but_v(P):
+    """Original ADOPT order, step 0 with non-finite gradients: v = g_0^2
+    (NaN or Inf where g_0 is), u and x bit-identical to their initial
+    values on every replica, averaged or not."""
+    for period in (0, 1):
+        w = workload_dict([1000, 37], 4, base="adopt", betas=(0.9, 0.99), beta2=0.9999, px=period,
+                          pu=period, pv=period, clip="elementwise")
+        w["opt"]["adopt_prev_v"] = True
+        lay = W.layout(w["shapes"])
+        idx = np.arange(lay["n_padded"])
+        eng = P.MTDAO(w["opt"], 4, w["shapes"])
+        x0 = G.init_params(w, lay, SEED_I, idx)
+        eng.set_params(torch.from_numpy(x0).cuda())
+        g = host_grads(w, lay, SEED_G, 0, idx)
+        g[0, 5], g[1, 9], g[2, 40] = np.nan, np.inf, -np.inf
+        eng.step(to_dev(g, "f32"), 2.0 ** -8, eng.sync_due())
+        torch.cuda.synchronize()
+        st = gpu_states(eng, w["opt"])
+        assert np.array_equal(st["x"], np.broadcast_to(x0, st["x"].shape))
+        for j in (1, 2):
+            assert not np.any(st["u%d" % j]), j
+        want = (g.astype(np.float32) ** 2)
+        if period == 1:
+            # averaged at the end of step 0: a column with a non-finite
+            # replica value is non-finite on every replica, the others hold
+            # the replica mean of g_0^2
+            nonfin = ~np.isfinite(want).all(axis=0)
+            assert np.array_equal(~np.isfinite(st["v"]), np.broadcast_to(nonfin, st["v"].shape))
+            mean = want[:, ~nonfin].astype(np.float64).mean(axis=0)
+            assert np.allclose(st["v"][:, ~nonfin], mean[None, :], rtol=1e-6, atol=0)
+        else:
+            assert np.array_equal(st["v"], want, equal_nan=True)
+        eng.close()
 
 
 def test_error_codes(P, monkeypatch):
@@ -351,6 +493,21 @@ def test_error_codes(P, monkeypatch):
     with pytest.raises(P.MTDAOError) as e:
         P.mtdao_sync(eng.h, 1 << 5)
     assert e.value.code == P.ERR_INVALID
+    # double outputs must be 8-byte aligned; refused before any launch
+    outs = torch.zeros(64, dtype=torch.float64, device="cuda")
+    bad = outs.data_ptr() + 4
+    for call in (lambda: P.mtdao_grad_sqnorm(eng.h, g.data_ptr(), P.F32, bad),
+                 lambda: P.mtdao_grad_nonfinite(eng.h, g.data_ptr(), P.F32, bad),
+                 lambda: P.mtdao_sync_stats(eng.h, 1, bad)):
+        with pytest.raises(P.MTDAOError) as e:
+            call()
+        assert e.value.code == P.ERR_ALIGN
+    P.mtdao_track_anchor(eng.h, 1)
+    with pytest.raises(P.MTDAOError) as e:
+        P.mtdao_pseudo_grad_stats(eng.h, 0, bad)
+    assert e.value.code == P.ERR_ALIGN
+    P.mtdao_track_anchor(eng.h, 0)
+    torch.cuda.synchronize()
     assert eng.t == 0
     eng.close()
     free0 = torch.cuda.mem_get_info()[0]

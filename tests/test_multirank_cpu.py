@@ -89,6 +89,10 @@ def test_reference_arm_json_line():
     assert d["config"]["workload"] == "decoder_1b"
     cb = d["cpu_baseline"]
     assert cb["kind"] == "oracle" and cb["cores"] >= 1 and cb["sample"] and cb["value"] == d["value"]
+    assert cb["cores"] == len(os.sched_getaffinity(0))          # every host core
+    # ms_per_step is the measured time of a step of the sample, which ran:
+    # well below a minute, not a full-size round extrapolated from it
+    assert 0 < d["ms_per_step"] < 60e3
     e = d["e2e"]
     assert e["value"] == d["value"] and e["unit"] == d["unit"]
     assert e["h2d_bytes_per_step"] == 0 and e["d2h_bytes_per_step"] == 0

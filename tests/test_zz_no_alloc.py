@@ -6,11 +6,13 @@ or they hold no handle because creating one allocates).
 The entry point keeps its partial sums in a fixed static device array.  This
 test calls it through the C ABI twice in a row on different inputs (different
 M, dtype and size, so the second call runs over slots the first one left
-behind) and checks each result against the handle-based mtdao_grad_sqnorm
-with the tolerance the other norm test uses (1e-6 relative).  It also checks
-that a repeated call leaves the device's free memory unchanged and that
-sizes beyond the limits are rejected.  Kept in a file that pytest collects
-last.
+behind) and checks each result against the handle-based mtdao_grad_sqnorm:
+both run the same grid in the same order, so the results must be equal bit
+for bit; both are also checked against an fp64 sum of squares with the
+tolerance the other norm tests use (1e-6 relative).  It also checks that a
+repeated call leaves the device's free memory unchanged and that sizes
+beyond the limits and a misaligned output are rejected.  Kept in a file that
+pytest collects last.
 """
 import numpy as np
 import pytest
@@ -53,7 +55,7 @@ def test_static_scratch_norm_matches_handle_version():
         P.mtdao_grad_sqnorm_static(g.data_ptr(), dt, M, n, out.data_ptr(), stream)
         torch.cuda.synchronize()
         got, want = out.cpu().numpy(), ref.cpu().numpy()
-        assert np.all(np.abs(got - want) <= TOL * np.abs(want)), (got, want)
+        assert np.array_equal(got.view(np.uint64), want.view(np.uint64)), (got, want)
         exact = np.sum(g_host.astype(np.float64) ** 2, axis=1)
         assert np.all(np.abs(got - exact) <= TOL * exact)
 
@@ -71,3 +73,8 @@ def test_static_scratch_norm_matches_handle_version():
             P.mtdao_grad_sqnorm_static(g.data_ptr(), P.F32, M, npad, out.data_ptr(), stream)
         assert e.value.code == P.ERR_INVALID
         assert P.mtdao_last_error(None)
+    # an output that is not 8-byte aligned is refused before any launch
+    with pytest.raises(P.MTDAOError) as e:
+        P.mtdao_grad_sqnorm_static(g.data_ptr(), P.F32, 2, n, out.data_ptr() + 4, stream)
+    assert e.value.code == P.ERR_ALIGN
+    torch.cuda.synchronize()
