@@ -10,7 +10,10 @@ Printed (rank 0, one JSON line): params/s = M * n * H / round time (whole
 job, all ranks), plus the roofline of the dominant kernel (the local-step
 kernel, timed per launch with CUDA events on its stream), the standalone
 sync kernel's bandwidth, an end-to-end figure through the host-buffer C-ABI
-call, and the CPU oracle timed on a bounded sample.
+call, and the CPU oracle timed on a bounded sample (one core and all the
+host's cores).  The default run also times the ~350M decoder list (ADOPT,
+bf16 gradients, M = 8, per-state periods K_x = 64, K_u = K_v = 16) in a
+child process and reports it under "workloads".
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
                   [--workload decoder_1b|gpt2_small|decoder_350m|tiny]
@@ -58,6 +61,8 @@ def parse_args():
                     help="flat-vector sweep: one JSON line per (n, M, N) with step, fused "
                          "step+sync and sync bandwidth, and the round rate for H in {1, 8, 64}")
     ap.add_argument("--sweep-log2n", default="20,24,27,30")
+    ap.add_argument("--second-workload", default="decoder_350m",
+                    help="workload timed in a child process after the main one ('' = none)")
     return ap.parse_args()
 
 
@@ -199,37 +204,95 @@ def parse_clock_samples(lines) -> dict:
 
 # --------------------------------------------------------------------- CPU oracle
 
-def oracle_sample_rate(w, n_sample: int, rounds: int = 1):
-    """Time the CPU oracle (as it stands, one thread) on n_sample elements of
-    every replica for `rounds` rounds of H local steps with their syncs.
-    Returns (params/s, seconds, description)."""
-    import numpy as np
+def host_cores() -> int:
+    """Host cores this process may run on."""
+    try:
+        return len(os.sched_getaffinity(0))
+    except AttributeError:
+        return os.cpu_count() or 1
 
-    from oracle.oracle import Oracle
-    from synth import generators as G
 
-    lay = W.layout(w["shapes"])
-    opt, M = w["opt"], w["M"]
-    H = round_len(opt)
-    idx = np.arange(n_sample, dtype=np.int64)
-    x0 = G.init_params(w, lay, W.INIT_SEED, idx).astype(np.float64)
-    g = np.stack([G.grads(w, lay, W.GRAD_SEED, m, 0, idx) for m in range(M)]).astype(np.float64)
-    o = Oracle(opt, M, n_sample, x0=x0)
-    spent = 0.0
-    t = 0
-    for _ in range(rounds):
-        for _ in range(H):
-            t0 = time.perf_counter()
-            o.step(t, opt["lr"], g)
-            spent += time.perf_counter() - t0
-            t += 1
-    t0 = time.perf_counter()
-    o.settle(t)
-    spent += time.perf_counter() - t0
-    rate = M * n_sample * H * rounds / spent
-    desc = ("%d replicas x first %d elements x %d round(s) of %d local steps with the round's "
-            "syncs; one resident gradient batch" % (M, n_sample, rounds, H))
-    return rate, spent, desc
+class OracleSlices:
+    """The CPU oracle, as it stands, on `threads` disjoint slices of a
+    workload's elements (n_per_thread consecutive elements of every replica
+    each; slice k starts at element k * n_per_thread).  Each slice is its own
+    oracle instance with all M replicas, run by its own thread (the oracle's
+    C calls release the interpreter lock).  Without global-norm clipping the
+    elements of the method are independent, so the slices together compute
+    exactly what one oracle over all of them would; nothing in the oracle is
+    changed or tuned for this."""
+
+    def __init__(self, w, n_per_thread: int, threads: int):
+        import concurrent.futures as cf
+
+        import numpy as np
+
+        from oracle.oracle import Oracle
+        from synth import generators as G
+
+        assert w["opt"].get("clip_mode", "none") != "global_norm", \
+            "global-norm clipping couples the elements of a replica"
+        self.w, self.opt, self.M = w, w["opt"], w["M"]
+        self.H = round_len(self.opt)
+        self.n_per, self.threads = n_per_thread, threads
+        lay = W.layout(w["shapes"])
+        self.slices = []
+        for k in range(threads):
+            idx = np.arange(k * n_per_thread, (k + 1) * n_per_thread, dtype=np.int64)
+            x0 = G.init_params(w, lay, W.INIT_SEED, idx).astype(np.float64)
+            g = np.stack([G.grads(w, lay, W.GRAD_SEED, m, 0, idx) for m in range(self.M)]).astype(np.float64)
+            self.slices.append((Oracle(self.opt, self.M, n_per_thread, x0=x0), g))
+        self.pool = cf.ThreadPoolExecutor(max_workers=threads)
+        self.t = 0
+
+    def round(self) -> float:
+        """One round (H local steps of every slice, all replicas); returns
+        its wall time in seconds.  The oracle performs a round's averages
+        at the start of the next round's first step (Algorithm 1's form)."""
+        t, H, lr = self.t, self.H, self.opt["lr"]
+
+        def work(item):
+            o, g = item
+            for s in range(H):
+                o.step(t + s, lr, g)
+
+        t0 = time.perf_counter()
+        list(self.pool.map(work, self.slices))
+        dt = time.perf_counter() - t0
+        self.t += H
+        return dt
+
+    def units_per_round(self) -> int:
+        return self.M * self.n_per * self.threads * self.H
+
+    def describe(self) -> str:
+        return ("%d thread(s) x %d elements of every replica (M = %d, elements [0, %d) of the "
+                "workload) x rounds of %d local steps with their averages; one resident gradient "
+                "batch" % (self.threads, self.n_per, self.M, self.threads * self.n_per, self.H))
+
+    def close(self):
+        self.pool.shutdown()
+
+
+def cpu_baseline(w) -> dict:
+    """The oracle timed on the host: one round on one core (2^21 elements
+    of every replica, ~13 s on a Grace core) and one round on every core
+    (2^19 elements per core)."""
+    one = OracleSlices(w, 1 << 21, 1)
+    s1 = one.round()
+    r1 = one.units_per_round() / s1
+    d1 = one.describe()
+    one.close()
+    del one
+    cores = host_cores()
+    allc = OracleSlices(w, 1 << 19, cores)
+    sa = allc.round()
+    ra = allc.units_per_round() / sa
+    da = allc.describe()
+    allc.close()
+    return {"value": ra, "unit": "params/s", "cores": cores, "kind": "oracle", "sample": da,
+            "seconds": round(sa, 2),
+            "one_core": {"value": r1, "unit": "params/s", "cores": 1, "sample": d1, "seconds": round(s1, 2)}}
 
 
 def run_reference(args):
@@ -237,16 +300,15 @@ def run_reference(args):
     if rank != 0:
         return 0
     w = W.get(args.workload)
-    n_sample = 1 << 18
+    cores = host_cores()
+    sl = OracleSlices(w, 1 << 18, cores)
     for _ in range(max(args.warmup, 0)):
-        oracle_sample_rate(w, n_sample)
-    rates, total = [], 0.0
-    for _ in range(args.steps):
-        r, s, desc = oracle_sample_rate(w, n_sample)
-        rates.append(r)
-        total += s
-    value = statistics.median(rates)
-    H = round_len(w["opt"])
+        sl.round()
+    secs = [sl.round() for _ in range(args.steps)]
+    sl.close()
+    med = statistics.median(secs)
+    value = sl.units_per_round() / med
+    desc = sl.describe()
     line = {
         "impl": "reference",
         "metric": "fused MT-DAO step params/s (replica-parameter updates per second, syncs included)",
@@ -255,14 +317,17 @@ def run_reference(args):
         "n_gpus": args.gpus,
         "steps": args.steps,
         "warmup": args.warmup,
-        "ms_per_step": 1e3 * W.layout(w["shapes"])["n_padded"] * w["M"] * H / value,
+        # measured: one step = one round of the bounded sample below (not the
+        # full workload, which the oracle would take hours for)
+        "ms_per_step": 1e3 * med,
+        "ms_per_step_measured_on": "the sample (%d replica-element updates per round)" % sl.units_per_round(),
         "higher_is_better": True,
         "scaling": "weak",
         "vs_baseline": None,
         "dtype": "f64",
         "data": "synthetic",
         "config": {"workload": w["name"], "desc": w["desc"], "sample": desc},
-        "cpu_baseline": {"value": value, "unit": "params/s", "cores": 1, "kind": "oracle",
+        "cpu_baseline": {"value": value, "unit": "params/s", "cores": cores, "kind": "oracle",
                          "sample": desc},
         "e2e": {"value": value, "unit": "params/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
         "gpu_launches": 0,
@@ -427,9 +492,14 @@ def run_ours(args):
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        rate, spent, desc = oracle_sample_rate(w, 1 << 21)      # ~13 s of one host core
-        cpu = {"value": rate, "unit": "params/s", "cores": 1, "kind": "oracle", "sample": desc,
-               "seconds": round(spent, 2)}
+        cpu = cpu_baseline(w)
+
+    # the second named workload, in a fresh process (its allocations are
+    # not the first ones after a large free, and it does not share this
+    # process's state); this process keeps its memory meanwhile
+    second = None
+    if rank == 0 and world == 1 and args.second_workload and args.second_workload != w["name"]:
+        second = run_child_workload(args.second_workload, args.steps, args.warmup)
 
     traffic = measured_traffic(step_kernel_name(opt, w["grad_dtype"]), M * n)
     line = {
@@ -448,6 +518,7 @@ def run_ours(args):
         "config": {
             "workload": w["name"], "desc": w["desc"], "M": M, "n_padded": n, "n_mom": opt["n_mom"],
             "base": opt["base"], "grad_dtype": w["grad_dtype"], "local_steps_per_step": H,
+            "periods": {"x": opt["period_x"], "u": list(opt["period_u"]), "v": opt.get("period_v", 0)},
             "step": "one communication round: H local steps, the due averages fused into the last",
             "grads": "one resident synthetic gradient batch per replica, reused every local step",
             "l2": ("L2 flushed before every launch; time = sum of launch times" if small else
@@ -484,6 +555,7 @@ def run_ours(args):
                      "frac": achieved / peak, "traffic": traffic, "peak_kind": peak_kind,
                      "kernel": step_kernel_name(opt, w["grad_dtype"])},
         "cpu_baseline": cpu,
+        "workloads": second,
         "e2e": e2e,
         "gpu_launches": args.steps * H * (3 if opt.get("clip_mode") == "global_norm" else 1),
         "clocks": clocks,
@@ -494,6 +566,39 @@ def run_ours(args):
     if dist is not None:
         dist.destroy_process_group()
     return 0
+
+
+def run_child_workload(name: str, steps: int, warmup: int):
+    """Run this benchmark on workload `name` in a child process (no e2e, no
+    CPU baseline) and summarise its kernel and round figures."""
+    cmd = [sys.executable, os.path.abspath(__file__), "--workload", name, "--steps", str(steps),
+           "--warmup", str(warmup), "--no-e2e", "--no-cpu-baseline", "--second-workload", ""]
+    env = {k: v for k, v in os.environ.items()
+           if k not in ("RANK", "WORLD_SIZE", "LOCAL_RANK", "LOCAL_WORLD_SIZE", "MASTER_ADDR", "MASTER_PORT")}
+    try:
+        r = subprocess.run(cmd, capture_output=True, text=True, timeout=900, env=env, cwd=ROOT)
+    except subprocess.TimeoutExpired:
+        return {name: {"error": "timed out"}}
+    lines = [ln for ln in r.stdout.splitlines() if ln.startswith("{")]
+    if r.returncode != 0 or not lines:
+        return {name: {"error": "exit %d: %s" % (r.returncode, r.stderr.strip().splitlines()[-1:])}}
+    c = json.loads(lines[-1])
+    cfg = c["config"]
+    return {name: {
+        "value": c["value"], "unit": c["unit"], "ms_per_step": c["ms_per_step"],
+        "step": cfg["step"], "local_steps_per_step": cfg["local_steps_per_step"],
+        "M": cfg["M"], "n_padded": cfg["n_padded"], "n_mom": cfg["n_mom"], "base": cfg["base"],
+        "grad_dtype": cfg["grad_dtype"], "periods": cfg.get("periods"),
+        "step_kernel": {k: c["step_kernel"][k] for k in ("ms_mean", "ms_median", "gbs", "bytes")},
+        "step_kernel_frac": c["roofline"]["frac"],
+        "sync_step_kernel": c["sync_step_kernel"],
+        "sync_kernel": {k: c["sync_kernel"][k] for k in ("ms_median", "gbs", "frac", "states")},
+        "sync_stats_kernel": c.get("sync_stats_kernel"),
+        "pseudo_grad_stats_kernel": c.get("pseudo_grad_stats_kernel"),
+        "grad_sqnorm_kernel": c.get("grad_sqnorm_kernel"),
+        "peak": c["roofline"]["peak"], "kernel": c["roofline"]["kernel"],
+        "gpu_launches": c["gpu_launches"], "clocks": c["clocks"],
+    }}
 
 
 def run_sweep(args):
