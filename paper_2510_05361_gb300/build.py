@@ -21,8 +21,8 @@ CSRC = os.path.join(PKG, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 OUT_DIR = os.path.join(PKG, "_build")
 LIB = os.path.join(OUT_DIR, "libmtdao.so")
-SOURCES = ["mtdao_api.cu", "reduce_kernels.cu", "step_adam.cu", "step_adopt.cu", "step_sgdm.cu",
-           "noalloc.cu"]
+SOURCES = ["mtdao_api.cu", "reduce_kernels.cu", "stats_wide.cu", "step_adam.cu", "step_adopt.cu",
+           "step_sgdm.cu", "noalloc.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ARCH + ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC",
                      "-prec-div=true", "-prec-sqrt=true", "-ftz=false",

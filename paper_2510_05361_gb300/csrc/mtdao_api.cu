@@ -505,16 +505,26 @@ static int refresh_anchor(mtdao_ctx *h, uint32_t mask) {
     return MTDAO_OK;
 }
 
-// Diagnostics kernels hold M replicas in registers up to this M; above it
-// they take two passes through a scratch vector.
+// Diagnostics kernels hold M replicas in registers up to this M; up to
+// kWideStatsM they stage all replicas of a span in shared memory (one
+// pass); above it they take two passes through a scratch vector.
 constexpr int kStatsRegisterM = 8;
+constexpr int kWideStatsM = 256;
+
+enum StatsPath { kStatsRegister, kStatsWide, kStatsGeneral };
+
+static StatsPath stats_path(const mtdao_ctx *h) {
+    return h->M <= kStatsRegisterM ? kStatsRegister : (h->M <= kWideStatsM ? kStatsWide : kStatsGeneral);
+}
 
 static int ensure_stats_workspace(mtdao_ctx *h) {
-    const bool general = h->M > kStatsRegisterM;
+    const StatsPath path = stats_path(h);
+    const bool general = path == kStatsGeneral;
     if (h->stats_partial != nullptr && (!general || h->stats_mean != nullptr)) return MTDAO_OK;
     if (h->stats_partial == nullptr) {
-        const size_t cap = general ? general_stats_partial_capacity(h->num_sms, h->M)
-                                   : sync_stats_partial_capacity(h->num_sms, h->n_states, h->M);
+        const size_t cap = path == kStatsGeneral ? general_stats_partial_capacity(h->num_sms, h->M)
+                           : path == kStatsWide  ? wide_stats_partial_capacity(h->num_sms, h->n_states, h->M)
+                                                 : sync_stats_partial_capacity(h->num_sms, h->n_states, h->M);
         cudaError_t e = cudaMalloc(reinterpret_cast<void **>(&h->stats_partial), cap * sizeof(double));
         if (e != cudaSuccess) {
             cudaGetLastError();
@@ -709,10 +719,14 @@ extern "C" int mtdao_sync_stats(mtdao_handle h, uint32_t mask, double *stats_dev
     a.M = h->M;
     for (int s = 0; s < h->n_states; ++s)
         if (mask & (1u << s)) a.sel[a.n_sel++] = s;
-    cudaError_t e = h->M > kStatsRegisterM
-                        ? launch_sync_stats_general(a, h->num_sms, h->stats_mean, h->stats_partial, h->stats_cap,
-                                                    stats_dev, h->stream)
-                        : launch_sync_stats(a, h->num_sms, h->stats_partial, h->stats_cap, stats_dev, h->stream);
+    const StatsPath path = stats_path(h);
+    cudaError_t e =
+        path == kStatsGeneral
+            ? launch_sync_stats_general(a, h->num_sms, h->stats_mean, h->stats_partial, h->stats_cap, stats_dev,
+                                        h->stream)
+        : path == kStatsWide ? launch_sync_stats_wide(a, h->num_sms, h->stats_partial, h->stats_cap, stats_dev,
+                                                      h->stream)
+                             : launch_sync_stats(a, h->num_sms, h->stats_partial, h->stats_cap, stats_dev, h->stream);
     if (e != cudaSuccess) return cuda_fail(h, e, "sync with diagnostics launch");
     return refresh_anchor(h, mask);
 }
@@ -759,12 +773,15 @@ extern "C" int mtdao_pseudo_grad_stats(mtdao_handle h, int32_t state, double *ou
     if (int rc = select_device(h)) return rc;
     if (int rc = ensure_stats_workspace(h)) return rc;
     const float *x = h->arena + static_cast<int64_t>(state) * h->M * h->n_padded;
-    cudaError_t e = h->M > kStatsRegisterM
-                        ? launch_pseudo_grad_stats_general(x, h->anchor[state], h->n_padded, h->M, h->num_sms,
-                                                           h->stats_mean, h->stats_partial, h->stats_cap,
-                                                           out_dev, h->stream)
-                        : launch_pseudo_grad_stats(x, h->anchor[state], h->n_padded, h->M, h->num_sms,
-                                                   h->stats_partial, h->stats_cap, out_dev, h->stream);
+    const StatsPath path = stats_path(h);
+    cudaError_t e =
+        path == kStatsGeneral
+            ? launch_pseudo_grad_stats_general(x, h->anchor[state], h->n_padded, h->M, h->num_sms, h->stats_mean,
+                                               h->stats_partial, h->stats_cap, out_dev, h->stream)
+        : path == kStatsWide ? launch_pseudo_grad_stats_wide(x, h->anchor[state], h->n_padded, h->M, h->num_sms,
+                                                             h->stats_partial, h->stats_cap, out_dev, h->stream)
+                             : launch_pseudo_grad_stats(x, h->anchor[state], h->n_padded, h->M, h->num_sms,
+                                                        h->stats_partial, h->stats_cap, out_dev, h->stream);
     if (e != cudaSuccess) return cuda_fail(h, e, "change diagnostics launch");
     return MTDAO_OK;
 }

@@ -23,7 +23,8 @@ constexpr int kNormThreads = 256;    // threads per block of the norm reduction
 // fma(c, target, fma(-c, s, s)): beta * s is formed exactly inside the
 // inner fma and rounded once, so beta = 0 gives the target exactly however
 // large s was.  The second moment is fma(c * g, g, fma(-c, s, s)) in the
-// same way, so beta_2 = 0 gives g^2.
+// same way, so beta_2 = 0 gives g^2.  An infinite s skips the inner fma
+// (ema_decay): beta * s is then s, not the fma's inf - inf.
 struct StepScalars {
     float neg_lr;                    // -eta_t
     float c1[MTDAO_MAX_MOM];         // 1 - beta_{1,j}
@@ -62,7 +63,7 @@ cudaError_t launch_step(int base, int n_mom, int grad_dtype, bool clip, const St
                         int num_sms, cudaStream_t stream);
 
 // Local step with the replica average of the states in a.sync_mask fused
-// into the same pass.  For 2 <= M <= 8 and M = 16; returns cudaErrorNotSupported
+// into the same pass.  For 2 <= M <= 256; returns cudaErrorNotSupported
 // otherwise (the caller then runs launch_step followed by launch_sync).
 cudaError_t launch_step_sync(int base, int n_mom, int grad_dtype, bool clip, const StepArgs &a,
                              int num_sms, cudaStream_t stream);
@@ -83,6 +84,17 @@ size_t sync_stats_partial_capacity(int num_sms, int n_states, int M);
 cudaError_t launch_sync_stats(const SyncArgs &a, int num_sms, double *partial, size_t partial_cap,
                               double *stats, cudaStream_t stream);
 
+// One-pass diagnostics for 2 <= M <= 256 (the wide layout of the fused
+// step): same outputs as launch_sync_stats / launch_pseudo_grad_stats, the
+// averaged states bit-identical to launch_sync's.  Workspace: partial needs
+// wide_stats_partial_capacity() doubles.
+size_t wide_stats_partial_capacity(int num_sms, int n_states, int M);
+cudaError_t launch_sync_stats_wide(const SyncArgs &a, int num_sms, double *partial, size_t partial_cap,
+                                   double *stats, cudaStream_t stream);
+cudaError_t launch_pseudo_grad_stats_wide(const float *x, const float *anchor, int64_t n, int M, int num_sms,
+                                          double *partial, size_t partial_cap, double *stats,
+                                          cudaStream_t stream);
+
 // Per-replica sum of squares of the gradient: partial sums into
 // partial[M][blocks_per_replica], then out[m] (double) and, when
 // clip_scale != nullptr, clip_scale[m] = min(1, rho / (sqrt(out[m]) + 1e-6)).
@@ -91,8 +103,8 @@ cudaError_t launch_grad_sqnorm(const void *grads, int grad_dtype, int32_t M, int
                                int blocks_per_replica, double *partial, double *out,
                                float *clip_scale, double rho, cudaStream_t stream);
 
-// Diagnostics for any M (two passes per state through a [n_padded] fp32
-// scratch that holds the replica mean; see reduce_kernels.cu).  Same
+// Diagnostics for any M, used above 256 (two passes per state through a
+// [n_padded] fp32 scratch that holds the replica mean; see reduce_kernels.cu).  Same
 // outputs as launch_sync_stats / launch_pseudo_grad_stats; the averaged
 // states are bit-identical to launch_sync's.  Workspace: partial needs
 // general_stats_partial_capacity() doubles.

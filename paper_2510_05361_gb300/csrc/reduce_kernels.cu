@@ -17,6 +17,7 @@
 #include <type_traits>
 
 #include "mtdao_internal.h"
+#include "kahan.cuh"
 #include "replica_mean.cuh"
 #include "step_kernels.cuh"
 
@@ -47,6 +48,7 @@ __global__ void __launch_bounds__(kThreads) sync_kernel(const SyncArgs a) {
             to_array(ld_state(base + e), s0);
             DiffSum pa[4] = {DiffSum(s0[0]), DiffSum(s0[1]), DiffSum(s0[2]), DiffSum(s0[3])};
             DiffSum pb[4] = {DiffSum(s0[0]), DiffSum(s0[1]), DiffSum(s0[2]), DiffSum(s0[3])};
+            float plain[4] = {s0[0], s0[1], s0[2], s0[3]};
             const int h = M / 2;
             for (int m = 1; m < M; ++m) {
                 float r[4];
@@ -55,10 +57,13 @@ __global__ void __launch_bounds__(kThreads) sync_kernel(const SyncArgs a) {
                 for (int k = 0; k < 4; ++k) {
                     if (m < h) pa[k].add(r[k]);
                     else pb[k].add(r[k]);
+                    plain[k] += r[k];
                 }
             }
 #pragma unroll
-            for (int k = 0; k < 4; ++k) mean[k] = replica_mean_from_parts(s0[k], pa[k].partial(), pb[k].partial(), Mf);
+            for (int k = 0; k < 4; ++k)
+                mean[k] = mean_or_plain(replica_mean_from_parts(s0[k], pa[k].partial(), pb[k].partial(), Mf),
+                                        plain[k], Mf);
         }
         const float4 mv = from_array(mean);
         for (int m = 0; m < M; ++m) st_state(base + m * n + e, mv);
@@ -86,12 +91,6 @@ cudaError_t launch_sync_t(const SyncArgs &a, int num_sms, cudaStream_t stream) {
     dim3 grid(static_cast<unsigned>(gx), static_cast<unsigned>(a.n_sel));
     sync_kernel<MT><<<grid, kThreads, 0, stream>>>(a);
     return cudaGetLastError();
-}
-
-__device__ __forceinline__ double warp_sum(double v) {
-#pragma unroll
-    for (int off = 16; off > 0; off >>= 1) v += __shfl_down_sync(0xffffffffu, v, off);
-    return v;
 }
 
 // Deterministic block sum of one double per thread; result valid in thread 0.
@@ -233,21 +232,6 @@ __global__ void __launch_bounds__(kNormThreads) sqnorm_finalize_kernel(const dou
 }
 
 // ---------------------------------------------------------------- sync + diagnostics
-
-// fp32 accumulator with Kahan compensation; value() folds the compensation
-// in at double precision.
-struct Kahan {
-    float s = 0.0f, c = 0.0f;
-    __device__ __forceinline__ void add(float y) {
-        y -= c;
-        const float t = s + y;
-        c = (t - s) - y;
-        s = t;
-    }
-    __device__ __forceinline__ double value() const {
-        return static_cast<double>(s) - static_cast<double>(c);
-    }
-};
 
 // Replica average of the selected states (exactly as sync_kernel) plus, in
 // the same pass over the M replicas, per state and block the partial sums of
@@ -462,6 +446,7 @@ __device__ __forceinline__ float4 replica_mean4(const float *s, int64_t n, int M
     to_array(ld_state(s + e), s0);
     DiffSum pa[4] = {DiffSum(s0[0]), DiffSum(s0[1]), DiffSum(s0[2]), DiffSum(s0[3])};
     DiffSum pb[4] = {DiffSum(s0[0]), DiffSum(s0[1]), DiffSum(s0[2]), DiffSum(s0[3])};
+    float plain[4] = {s0[0], s0[1], s0[2], s0[3]};
     const int h = M / 2;
     for (int m = 1; m < M; m += 4) {          // four replicas' loads in flight, added in order
         float r[4][4];
@@ -475,13 +460,16 @@ __device__ __forceinline__ float4 replica_mean4(const float *s, int64_t n, int M
             for (int k = 0; k < 4; ++k) {
                 if (m + u < h) pa[k].add(r[u][k]);
                 else pb[k].add(r[u][k]);
+                plain[k] += r[u][k];
             }
         }
     }
     float mean[4];
 #pragma unroll
     for (int k = 0; k < 4; ++k)
-        mean[k] = replica_mean_from_parts(s0[k], pa[k].partial(), pb[k].partial(), static_cast<float>(M));
+        mean[k] = mean_or_plain(
+            replica_mean_from_parts(s0[k], pa[k].partial(), pb[k].partial(), static_cast<float>(M)), plain[k],
+            static_cast<float>(M));
     return from_array(mean);
 }
 

@@ -13,6 +13,15 @@
 // M = 1024).  The two parts let a kernel hold the replicas of one element
 // in two lanes (replicas 0 .. h-1 and h .. M-1) and still produce exactly
 // the value a single thread computes.
+//
+// Non-finite values: the compensated sum turns one infinite replica value
+// into NaN (inf - inf inside the compensation), where the mean of the
+// method, sum_m s_m / M, is +-inf when the values hold infinities of one
+// sign only.  So a NaN result is replaced by the plain fp32 sum of the M
+// values divided by M: NaN when a value is NaN or both infinities occur,
+// the infinity otherwise (the outcome does not depend on the order of the
+// sum).  Finite values reach this path only if a difference s_m - s_0
+// overflows (|s| near 3.4e38); the plain sum is then the fallback as well.
 #pragma once
 
 #include <cuda_runtime.h>
@@ -40,6 +49,11 @@ __device__ __forceinline__ float replica_mean_from_parts(float s0, float part_a,
     return q == 0.0f ? s0 : s0 + q;
 }
 
+// The compensated mean, or the plain one where it is NaN (see above).
+__device__ __forceinline__ float mean_or_plain(float mean, float plain_sum, float M) {
+    return mean != mean ? plain_sum / M : mean;
+}
+
 // The mean of M values held by one thread; get(m) returns replica m's value.
 template <int M, typename Get>
 __device__ __forceinline__ float replica_mean(Get get) {
@@ -50,7 +64,12 @@ __device__ __forceinline__ float replica_mean(Get get) {
     for (int m = 1; m < h; ++m) a.add(get(m));
 #pragma unroll
     for (int m = (h > 1 ? h : 1); m < M; ++m) b.add(get(m));
-    return replica_mean_from_parts(s0, a.partial(), b.partial(), static_cast<float>(M));
+    const float mean = replica_mean_from_parts(s0, a.partial(), b.partial(), static_cast<float>(M));
+    if (mean == mean) return mean;
+    float plain = s0;
+#pragma unroll
+    for (int m = 1; m < M; ++m) plain += get(m);
+    return plain / static_cast<float>(M);
 }
 
 // Same, for a replica count known only at run time.
@@ -61,7 +80,11 @@ __device__ __forceinline__ float replica_mean_rt(int M, Get get) {
     DiffSum a(s0), b(s0);
     for (int m = 1; m < h; ++m) a.add(get(m));
     for (int m = (h > 1 ? h : 1); m < M; ++m) b.add(get(m));
-    return replica_mean_from_parts(s0, a.partial(), b.partial(), static_cast<float>(M));
+    const float mean = replica_mean_from_parts(s0, a.partial(), b.partial(), static_cast<float>(M));
+    if (mean == mean) return mean;
+    float plain = s0;
+    for (int m = 1; m < M; ++m) plain += get(m);
+    return plain / static_cast<float>(M);
 }
 
 }  // namespace mtdao

@@ -88,6 +88,16 @@ __device__ __forceinline__ float step_acc_init(const StepScalars &sc, float g, f
     return BASE == MTDAO_BASE_ADOPT ? 0.0f : sc.cg * __fmul_rn(g, s);   // never contracted into an FMA
 }
 
+// beta * s for beta = 1 - c, rounded once: s - c * s in one fma, which keeps
+// beta's precision however close it is to 1.  For an infinite s the fma
+// would form inf - inf = NaN where beta * s is s itself (beta > 0), so an
+// infinite state stays infinite from one step to the next, as it does in
+// exact arithmetic; c = 1 (beta = 0) keeps the fma's NaN, which is 0 * inf.
+__device__ __forceinline__ float ema_decay(float c, float s) {
+    const float d = fmaf(-c, s, s);
+    return (fabsf(s) == __int_as_float(0x7f800000) && c < 1.0f) ? s : d;
+}
+
 // Update state `st` of one element of one replica for step t.
 //   g : raw gradient g_t^m          s : clip(g, rho) factor (1 when not clipping)
 //   cur : the state's value, updated in place
@@ -104,9 +114,9 @@ __device__ __forceinline__ void update_state(const StepScalars &sc, int st, floa
         float gn;
         if (sc.prev_v) {
             gn = g / (sqrtf(cur) + sc.eps);
-            cur = fmaf(__fmul_rn(sc.c2, g), g, fmaf(-sc.c2, cur, cur));
+            cur = fmaf(__fmul_rn(sc.c2, g), g, ema_decay(sc.c2, cur));
         } else {
-            cur = fmaf(__fmul_rn(sc.c2, g), g, fmaf(-sc.c2, cur, cur));
+            cur = fmaf(__fmul_rn(sc.c2, g), g, ema_decay(sc.c2, cur));
             gn = g / (sqrtf(cur) + sc.eps);
         }
         gn = gn > sc.clip_c ? sc.clip_c : (gn < -sc.clip_c ? -sc.clip_c : gn);  // keeps NaN
@@ -115,7 +125,7 @@ __device__ __forceinline__ void update_state(const StepScalars &sc, int st, floa
     } else if (st == 1 + N) {
         // Algorithm 1: v of the raw gradient, then the denominator
         // sqrt(v / b_v) + eps of the momenta's combination.
-        cur = fmaf(__fmul_rn(sc.c2, g), g, fmaf(-sc.c2, cur, cur));
+        cur = fmaf(__fmul_rn(sc.c2, g), g, ema_decay(sc.c2, cur));
         acc = acc / fmaf(sqrtf(cur), sc.sv, sc.eps);
     } else if (st == 0) {
         cur = fmaf(sc.neg_lr, acc, cur);                     // x - eta_t Delta
@@ -123,7 +133,7 @@ __device__ __forceinline__ void update_state(const StepScalars &sc, int st, floa
         // momentum u_j of clip(g) (Adam, SGDM) or of ADOPT's clamped g
         const int j = st - 1;
         const float target = BASE == MTDAO_BASE_ADOPT ? gt : __fmul_rn(g, s);
-        cur = fmaf(sc.c1[j], target, fmaf(-sc.c1[j], cur, cur));
+        cur = fmaf(sc.c1[j], target, ema_decay(sc.c1[j], cur));
         acc = fmaf(sc.k[j], cur, acc);
     }
 }

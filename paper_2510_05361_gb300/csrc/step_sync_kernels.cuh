@@ -10,6 +10,7 @@
 
 #include "replica_mean.cuh"
 #include "step_kernels.cuh"
+#include "step_sync_wide.cuh"
 
 namespace mtdao {
 
@@ -26,9 +27,10 @@ namespace mtdao {
 //   M = 16      : four groups of R = 4, V = 4; each part of the mean spans
 //                 two groups and its compensated sum is handed from one to
 //                 the next in replica order.
-// Other M take the plain step followed by the standalone average: 32
-// (eight groups of four lanes: 64-byte pieces of eight replica slabs per
-// load, slower than the separate average) and every M above 8 but 16.
+// Other M up to 64 take the block-staged kernel of step_sync_wide.cuh (a
+// lane-group shape for M = 32, eight groups of four lanes, loaded 64-byte
+// pieces of eight replica slabs and ran slower than the separate average);
+// above 64, the plain step followed by the standalone average.
 // The states are visited one after another (state_order); the next
 // state's loads are issued before the current state is updated and stored,
 // so two states' loads are in flight per lane within the 128-register cap.
@@ -131,7 +133,15 @@ __device__ __forceinline__ void store_replicas(float *state, int64_t n_padded, i
                 const float fin = part.partial();
                 const float a = __shfl_sync(0xffffffffu, fin, (H - 1) * S::kLanes + q);      // replicas 1 .. M/2-1
                 const float b = __shfl_sync(0xffffffffu, fin, (S::G - 1) * S::kLanes + q);   // replicas M/2 .. M-1
-                mean[k] = replica_mean_from_parts(s0, a, b, static_cast<float>(M));
+                // plain sum for the non-finite case: every group's lanes end with
+                // the same bits (a + b == b + a)
+                float plain = val[0][k];
+#pragma unroll
+                for (int r = 1; r < S::R; ++r) plain += val[r][k];
+#pragma unroll
+                for (int off = S::kLanes; off < 32; off <<= 1) plain += __shfl_xor_sync(0xffffffffu, plain, off);
+                mean[k] = mean_or_plain(replica_mean_from_parts(s0, a, b, static_cast<float>(M)), plain,
+                                        static_cast<float>(M));
             } else {
                 // replica 0 lives in group 0: its value is the reference of both parts
                 const float s0 = __shfl_sync(0xffffffffu, val[0][k], threadIdx.x & (S::kLanes - 1));
@@ -143,7 +153,12 @@ __device__ __forceinline__ void store_replicas(float *state, int64_t n_padded, i
                 const float other = __shfl_xor_sync(0xffffffffu, mine, S::kLanes);
                 const float a = grp == 0 ? mine : other;          // replicas 1 .. R-1
                 const float b = grp == 0 ? other : mine;          // replicas R .. M-1
-                mean[k] = replica_mean_from_parts(s0, a, b, static_cast<float>(M));
+                float plain = val[0][k];                          // for the non-finite case
+#pragma unroll
+                for (int r = 1; r < S::R; ++r) plain += val[r][k];
+                plain += __shfl_xor_sync(0xffffffffu, plain, S::kLanes);
+                mean[k] = mean_or_plain(replica_mean_from_parts(s0, a, b, static_cast<float>(M)), plain,
+                                        static_cast<float>(M));
             }
         }
 #pragma unroll
@@ -234,9 +249,9 @@ __global__ void __launch_bounds__(kThreads, 2) step_sync_kernel(const StepArgs a
                         float gn;
                         if (a.sc.prev_v) {
                             gn = gr / (sqrtf(cur[r][k]) + a.sc.eps);
-                            cur[r][k] = fmaf(__fmul_rn(a.sc.c2, gr), gr, fmaf(-a.sc.c2, cur[r][k], cur[r][k]));
+                            cur[r][k] = fmaf(__fmul_rn(a.sc.c2, gr), gr, ema_decay(a.sc.c2, cur[r][k]));
                         } else {
-                            cur[r][k] = fmaf(__fmul_rn(a.sc.c2, gr), gr, fmaf(-a.sc.c2, cur[r][k], cur[r][k]));
+                            cur[r][k] = fmaf(__fmul_rn(a.sc.c2, gr), gr, ema_decay(a.sc.c2, cur[r][k]));
                             gn = gr / (sqrtf(cur[r][k]) + a.sc.eps);
                         }
                         gn = gn > a.sc.clip_c ? a.sc.clip_c : (gn < -a.sc.clip_c ? -a.sc.clip_c : gn);
@@ -250,7 +265,7 @@ __global__ void __launch_bounds__(kThreads, 2) step_sync_kernel(const StepArgs a
 #pragma unroll
                     for (int k = 0; k < V; ++k) {
                         const float gr = g[r][k];
-                        cur[r][k] = fmaf(__fmul_rn(a.sc.c2, gr), gr, fmaf(-a.sc.c2, cur[r][k], cur[r][k]));
+                        cur[r][k] = fmaf(__fmul_rn(a.sc.c2, gr), gr, ema_decay(a.sc.c2, cur[r][k]));
                         acc[r][k] = acc[r][k] / fmaf(sqrtf(cur[r][k]), a.sc.sv, a.sc.eps);
                     }
             } else if (st == 0) {
@@ -266,7 +281,7 @@ __global__ void __launch_bounds__(kThreads, 2) step_sync_kernel(const StepArgs a
                     for (int k = 0; k < V; ++k) {
                         const float target =
                             BASE == MTDAO_BASE_ADOPT ? gt[r][k] : __fmul_rn(g[r][k], s[r]);
-                        cur[r][k] = fmaf(a.sc.c1[j], target, fmaf(-a.sc.c1[j], cur[r][k], cur[r][k]));
+                        cur[r][k] = fmaf(a.sc.c1[j], target, ema_decay(a.sc.c1[j], cur[r][k]));
                         acc[r][k] = fmaf(a.sc.k[j], cur[r][k], acc[r][k]);
                     }
             }
@@ -310,7 +325,7 @@ cudaError_t launch_step_sync_m(const StepArgs &a, int num_sms, cudaStream_t st) 
         case 7: return launch_step_sync_t<BASE, N, GDT, CLIP, 7>(a, num_sms, st);
         case 8: return launch_step_sync_t<BASE, N, GDT, CLIP, 8>(a, num_sms, st);
         case 16: return launch_step_sync_t<BASE, N, GDT, CLIP, 16>(a, num_sms, st);
-        default: return cudaErrorNotSupported;
+        default: return launch_step_sync_wide<BASE, N, GDT, CLIP>(a, st);
     }
 }
 

@@ -71,7 +71,7 @@ RAGGED = [1, 7, 300, 4099, 2560, 13]
 @pytest.mark.parametrize("gdt", ["f32", "bf16"])
 @pytest.mark.parametrize("N", [1, 2, 3, 4])
 @pytest.mark.parametrize("base", ["adam", "adopt", "sgdm"])
-@pytest.mark.parametrize("M", [2, 3, 4, 5, 6, 7, 8, 16, 32])
+@pytest.mark.parametrize("M", [2, 3, 4, 5, 6, 7, 8, 12, 16, 32, 64])
 def test_step_and_sync_parity_matrix(P, base, N, gdt, M):
     betas = W.SWEEP_BETAS[:N]
     w = workload_dict(RAGGED, M, base=base, betas=betas, beta2=0.9999 if base == "adopt" else 0.999,
@@ -96,7 +96,7 @@ def test_replica_counts(P, M):
 
 
 @pytest.mark.parametrize("gdt", ["f32", "bf16"])
-@pytest.mark.parametrize("M", [2, 3, 4, 5, 6, 7, 8, 16, 32])
+@pytest.mark.parametrize("M", [2, 3, 4, 5, 6, 7, 8, 9, 12, 16, 17, 24, 32, 33, 64, 100, 128, 200, 256])
 def test_fused_sync_is_bitwise_equal_to_separate_sync(P, M, gdt):
     for base in ("adam", "adopt", "sgdm"):
         w = workload_dict(RAGGED, M, base=base, betas=(0.9, 0.99, 0.5), px=3, pu=[2, 3, 4], pv=2,
@@ -110,7 +110,7 @@ def test_fused_sync_is_bitwise_equal_to_separate_sync(P, M, gdt):
         b.close()
 
 
-@pytest.mark.parametrize("M", [3, 4, 5, 7, 8, 16])
+@pytest.mark.parametrize("M", [3, 4, 5, 7, 8, 12, 16, 32])
 @pytest.mark.parametrize("gdt", ["f32", "bf16"])
 @pytest.mark.parametrize("base", ["adam", "sgdm"])
 def test_global_norm_clip_parity(P, base, gdt, M):
@@ -315,6 +315,53 @@ def test_sync_kernel_parity_and_invariants(P):
     eng.close()
 
 
+@pytest.mark.parametrize("path", ["sync", "stats", "fused"])
+@pytest.mark.parametrize("M", [2, 3, 4, 8, 12, 16, 300])
+def test_mean_of_nonfinite_values(P, M, path):
+    """The worker mean of values that hold infinities is the infinity when
+    they have one sign only, NaN when both signs or a NaN occur (the mean
+    sum_m s_m / M of the method), in the plain and the diagnostics average
+    and in the fused step (u_1 = beta u_1 with a zero gradient keeps the
+    values' classes).  Finite columns keep the compensated mean."""
+    if path == "fused" and M > 256:
+        pytest.skip("the fused average covers M <= 256")
+    shapes = [1024]
+    w = workload_dict(shapes, M, betas=(0.9, 0.99))
+    eng = P.MTDAO(w["opt"], M, shapes)
+    n = eng.n_padded
+    rng = np.random.default_rng(M)
+    vals = rng.standard_normal((M, n)).astype(np.float32)
+    vals[M - 1, 0] = np.inf                  # one +inf
+    vals[M // 2, 1] = -np.inf                # one -inf
+    vals[0, 2], vals[M - 1, 2] = np.inf, -np.inf
+    vals[1 % M, 3] = np.nan
+    vals[:, 4] = np.inf                      # every replica +inf
+    vals[0, 5] = -np.inf                     # the reference replica
+    u1 = 1
+    eng.state_view(u1).copy_(torch.from_numpy(vals).cuda())
+    if path == "sync":
+        eng.sync(1 << u1)
+        expect = vals.astype(np.float64).mean(0)
+    elif path == "stats":
+        eng.sync_stats(1 << u1)
+        expect = vals.astype(np.float64).mean(0)
+    else:
+        g = torch.zeros((M, n), device="cuda")
+        eng.step(g, 1e-3, 1 << u1)
+        beta = w["opt"]["beta1"][0]
+        expect = (beta * vals.astype(np.float64)).mean(0)
+    torch.cuda.synchronize()
+    got = eng.state_view(u1).cpu().numpy()
+    ref = np.broadcast_to(expect.astype(np.float32), (M, n))
+    assert np.array_equal(np.isnan(got), np.isnan(ref))
+    assert np.array_equal(np.isposinf(got), np.isposinf(ref))
+    assert np.array_equal(np.isneginf(got), np.isneginf(ref))
+    assert np.all(got == got[0:1]) or np.all(np.isnan(got) == np.isnan(got[0:1]))
+    fin = np.isfinite(ref)
+    assert np.allclose(got[fin], ref[fin], rtol=1e-5, atol=1e-6)
+    eng.close()
+
+
 @pytest.mark.parametrize("M", [1, 3, 4, 6, 8])
 def test_sync_identity_on_identical_replicas(P, M):
     w = workload_dict([777, 4096], M, betas=(0.9,))
@@ -391,18 +438,20 @@ NONFINITE_VARIANTS = {
 }
 
 
+@pytest.mark.parametrize("M", [4, 12])
 @pytest.mark.parametrize("t_plant", [0, 2])
 @pytest.mark.parametrize("sync", ["plain", "fused_every2", "fused_every1"])
 @pytest.mark.parametrize("gdt", ["f32", "bf16"])
 @pytest.mark.parametrize("variant", sorted(NONFINITE_VARIANTS))
-def test_nonfinite_gradients_propagate_like_the_oracle(P, variant, gdt, sync, t_plant):
-    """NaN, +Inf and -Inf gradients planted in three of four replicas at
+def test_nonfinite_gradients_propagate_like_the_oracle(P, variant, gdt, sync, t_plant, M):
+    """NaN, +Inf and -Inf gradients planted in three of M replicas at
     step 0 or 2, with no average, the fused average every second step, or
     every step: the NaN/Inf positions of every state equal the oracle's and
     the finite values agree within the tolerance.  The original ADOPT order
     (step 0 only sets v = g_0^2, Algorithm 2 read as the original method)
-    must leave u and x finite when step 0's gradient is not."""
-    M = 4
+    must leave u and x finite when step 0's gradient is not.  An infinite
+    state stays infinite at the next steps (beta * inf = inf), M = 12 runs
+    the fused average of the block-staged kernel."""
     period = {"plain": 0, "fused_every2": 2, "fused_every1": 1}[sync]
     kw = dict(NONFINITE_VARIANTS[variant])
     w = workload_dict([1000, 37], M, betas=(0.9, 0.99), px=period, pu=period, pv=period, gdt=gdt,
@@ -431,14 +480,12 @@ def test_nonfinite_gradients_propagate_like_the_oracle(P, variant, gdt, sync, t_
     torch.cuda.synchronize()
     got, ref = gpu_states(eng, w["opt"]), o.states()
     compare(got, ref)                    # includes: non-finite positions are equal
-    if sync == "plain":
-        # no average: NaN and each sign of Inf where the oracle has them (after
-        # an average the compensated mean turns an infinite replica value into
-        # NaN, where an fp64 mean keeps the infinity; still non-finite)
-        for k in ref:
-            assert np.array_equal(np.isnan(got[k]), np.isnan(ref[k])), k
-            assert np.array_equal(np.isposinf(got[k]), np.isposinf(ref[k])), k
-            assert np.array_equal(np.isneginf(got[k]), np.isneginf(ref[k])), k
+    # NaN and each sign of Inf where the oracle has them, averages included
+    # (the mean of values holding infinities of one sign is that infinity)
+    for k in ref:
+        assert np.array_equal(np.isnan(got[k]), np.isnan(ref[k])), k
+        assert np.array_equal(np.isposinf(got[k]), np.isposinf(ref[k])), k
+        assert np.array_equal(np.isneginf(got[k]), np.isneginf(ref[k])), k
     eng.close()
 
 
