@@ -507,9 +507,12 @@ static int refresh_anchor(mtdao_ctx *h, uint32_t mask) {
 
 // Diagnostics kernels hold M replicas in registers up to this M; up to
 // kWideStatsM they stage all replicas of a span in shared memory (one
-// pass); above it they take two passes through a scratch vector.
+// pass); above it they take two passes through a scratch vector (for
+// M = 128 and 256 the one-pass form, whose per-element mean is a chain of
+// M / 2 compensated additions, ran 2-4x slower than the plain average; the
+// two passes take 1.4x).
 constexpr int kStatsRegisterM = 8;
-constexpr int kWideStatsM = 256;
+constexpr int kWideStatsM = 64;
 
 enum StatsPath { kStatsRegister, kStatsWide, kStatsGeneral };
 

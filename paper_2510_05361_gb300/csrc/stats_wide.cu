@@ -11,8 +11,8 @@
 // sync diagnostics write the mean over it (the average itself), so a sync
 // with diagnostics moves the bytes of a plain sync.
 //
-// Sums are bit-reproducible: a position's four elements are summed in fp32,
-// each thread accumulates its positions with Kahan compensation, the P
+// Sums are bit-reproducible: a thread's 16 elements of a span are summed in
+// fp32, each thread accumulates its spans with Kahan compensation, the P
 // threads of a replica combine in fp64 by a fixed shuffle pattern, the
 // block writes one partial row, and a finalize kernel adds the rows in
 // block order.  The grid is persistent (spans strided by the grid), so the
@@ -37,6 +37,32 @@ __device__ __forceinline__ double replica_lanes_sum(double v, int P) {
     return v;
 }
 
+// float4 positions per thread and span: the span is S = 4 * P * kStatsVec
+// elements (rows of 128 bytes or more for every M up to 256).
+constexpr int kStatsVec = 4;
+constexpr int kStatsVecLog2 = 2;
+
+// 16-byte asynchronous global -> shared copies (cp.async, L2 only) and their
+// groups: a block copies the next span's tile while it works on this one.
+__device__ __forceinline__ void cp_async16(float *smem_dst, const float *gmem_src) {
+    const unsigned dst = static_cast<unsigned>(__cvta_generic_to_shared(smem_dst));
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;\n" ::"r"(dst), "l"(gmem_src) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;\n" ::"n"(N) : "memory"); }
+
+// Copies this thread's kStatsVec float4 positions of replica r of a span
+// (src: the replica's first element of the span) into its tile row, then
+// commits the group (an empty one when the span is past the end).
+__device__ __forceinline__ void fetch_row(bool live, float *dst, const float *src, int P) {
+    if (live) {
+#pragma unroll
+        for (int j = 0; j < kStatsVec; ++j) cp_async16(dst + 4 * P * j, src + 4 * P * j);
+    }
+    cp_async_commit();
+}
+
 // Sync diagnostics of the selected state blockIdx.y, partial row per block:
 //   q = 0          sum_m sum_i (s_m - s_bar)^2
 //   q = 1          sum_i s_bar^2
@@ -46,10 +72,12 @@ __device__ __forceinline__ double replica_lanes_sum(double v, int P) {
 // s_bar (the fp32 mean) is written over every replica.
 __global__ void __launch_bounds__(kWideMaxThreads) sync_stats_wide_kernel(const SyncArgs a, int log2_p,
                                                                           double *partial) {
-    extern __shared__ float smem[];
+    extern __shared__ __align__(16) float smem[];
+    constexpr int NV = kStatsVec;
     const int M = a.M;
     const int P = 1 << log2_p;
-    const int S = 4 * P;
+    const int log2_s = log2_p + 2 + kStatsVecLog2;
+    const int S = 1 << log2_s;
     const int Q = 2 + 2 * M;
     const int t = threadIdx.x;
     const int r = t >> log2_p;
@@ -58,49 +86,56 @@ __global__ void __launch_bounds__(kWideMaxThreads) sync_stats_wide_kernel(const 
     float *base = a.arena + static_cast<int64_t>(a.sel[blockIdx.y]) * a.stride;
     const int64_t n = a.n_padded;
     const int64_t n_spans = n / S;
-    float *tile = smem;                          // [M][S]
-    float *mean = smem + M * S;                  // [S]
+    float *tiles = smem;                         // [2][M][S]
+    float *mean = smem + 2 * M * S;              // [S]
     Kahan dev, sq, cross, msq;
 
-    for (int64_t span = blockIdx.x; span < n_spans; span += gridDim.x) {
-        const int64_t e = span * S + 4 * f;
-        float x[4] = {0.0f, 0.0f, 0.0f, 0.0f};
-        if (live) {
-            const float4 v = ld_state(base + r * n + e);
-            to_array(v, x);
-            *reinterpret_cast<float4 *>(tile + r * S + 4 * f) = v;
-        }
+    const int64_t first = blockIdx.x;
+    fetch_row(live && first < n_spans, tiles + r * S + 4 * f, base + r * n + first * S + 4 * f, P);
+    int buf = 0;
+    for (int64_t span = first; span < n_spans; span += gridDim.x, buf ^= 1) {
+        const int64_t next = span + gridDim.x;
+        fetch_row(live && next < n_spans, tiles + ((buf ^ 1) * M + r) * S + 4 * f,
+                  base + r * n + next * S + 4 * f, P);
+        cp_async_wait<1>();                      // this thread's copies of `span` have landed
+        __syncthreads();                         // ... and every thread's
+        const float *tile = tiles + buf * M * S;
+        tile_means(tile, M, log2_s, S, mean);
         __syncthreads();
-        tile_means(tile, M, S, S, mean);
-        __syncthreads();
         if (live) {
-            const float4 mv = *reinterpret_cast<const float4 *>(mean + 4 * f);
-            float mb[4];
-            to_array(mv, mb);
-            float p0 = 0.0f, p1 = 0.0f, p2 = 0.0f, p3 = 0.0f;
+            float p0 = 0.0f, p1 = 0.0f, p2 = 0.0f, p3 = 0.0f;   // this thread's 4 * NV elements
 #pragma unroll
-            for (int k = 0; k < 4; ++k) {
-                const float dv = x[k] - mb[k];
-                p0 = fmaf(dv, dv, p0);
-                p1 = fmaf(x[k], x[k], p1);
-                p2 = fmaf(x[k], mb[k], p2);
-                p3 = fmaf(mb[k], mb[k], p3);
+            for (int j = 0; j < NV; ++j) {
+                const int c = 4 * f + 4 * P * j;
+                float x[4], mb[4];
+                to_array(*reinterpret_cast<const float4 *>(tile + r * S + c), x);
+                const float4 mv = *reinterpret_cast<const float4 *>(mean + c);
+                to_array(mv, mb);
+#pragma unroll
+                for (int k = 0; k < 4; ++k) {
+                    const float dv = x[k] - mb[k];
+                    p0 = fmaf(dv, dv, p0);
+                    p1 = fmaf(x[k], x[k], p1);
+                    p2 = fmaf(x[k], mb[k], p2);
+                    p3 = fmaf(mb[k], mb[k], p3);
+                }
+                st_state(base + r * n + span * S + c, mv);
             }
             dev.add(p0);
             sq.add(p1);
             cross.add(p2);
             if (r == 0) msq.add(p3);
-            st_state(base + r * n + e, mv);
         }
-        __syncthreads();                         // the tile is reused by the next span
+        __syncthreads();                         // this tile and the means are rewritten next
     }
+    cp_async_wait<0>();
 
     // Per replica: its P lanes' sums; then one row of Q values.
     const double d = replica_lanes_sum(dev.value(), P);
     const double s2 = replica_lanes_sum(sq.value(), P);
     const double c2 = replica_lanes_sum(cross.value(), P);
     const double m2 = replica_lanes_sum(msq.value(), P);   // replica 0's lanes hold sum s_bar^2
-    double *red = reinterpret_cast<double *>(smem);        // [3][M] + 1, over the (now idle) tile
+    double *red = reinterpret_cast<double *>(smem);        // [3][M] + 1, over the (now idle) tiles
     if (live && f == 0) {
         red[r] = d;
         red[M + r] = s2;
@@ -131,50 +166,64 @@ __global__ void __launch_bounds__(kWideMaxThreads) sync_stats_wide_kernel(const 
 //   q = M + m      sum_i (x_m - a) * (x_bar - a)
 //   q = 2M         sum_i (x_bar - a)^2
 //   q = 2M + 1     sum_i a^2
+// The anchor's span travels with replica 0's row (one more tile row).
 __global__ void __launch_bounds__(kWideMaxThreads) pseudo_grad_stats_wide_kernel(const float *x,
                                                                                  const float *anchor,
                                                                                  int64_t n, int M, int log2_p,
                                                                                  double *partial) {
-    extern __shared__ float smem[];
+    extern __shared__ __align__(16) float smem[];
+    constexpr int NV = kStatsVec;
     const int P = 1 << log2_p;
-    const int S = 4 * P;
+    const int log2_s = log2_p + 2 + kStatsVecLog2;
+    const int S = 1 << log2_s;
     const int Q = 2 * M + 2;
     const int t = threadIdx.x;
     const int r = t >> log2_p;
     const int f = t & (P - 1);
     const bool live = r < M;
     const int64_t n_spans = n / S;
-    float *tile = smem;                          // [M][S]
-    float *mean = smem + M * S;                  // [S]
-    float *anc = mean + S;                       // [S]
+    const int R = M + 1;                         // tile rows: the replicas, then the anchor
+    float *tiles = smem;                         // [2][M + 1][S]
+    float *mean = smem + 2 * R * S;              // [S]
     Kahan loc2, cross, glob2, a2;
 
-    for (int64_t span = blockIdx.x; span < n_spans; span += gridDim.x) {
-        const int64_t e = span * S + 4 * f;
-        float xv[4] = {0.0f, 0.0f, 0.0f, 0.0f};
-        if (live) {
-            const float4 v = ld_state(x + r * n + e);
-            to_array(v, xv);
-            *reinterpret_cast<float4 *>(tile + r * S + 4 * f) = v;
-            if (r == 0)
-                *reinterpret_cast<float4 *>(anc + 4 * f) = __ldcs(reinterpret_cast<const float4 *>(anchor + e));
-        }
-        __syncthreads();
-        tile_means(tile, M, S, S, mean);
-        __syncthreads();
-        if (live) {
-            float mb[4], av[4];
-            to_array(*reinterpret_cast<const float4 *>(mean + 4 * f), mb);
-            to_array(*reinterpret_cast<const float4 *>(anc + 4 * f), av);
-            float p0 = 0.0f, p1 = 0.0f, p2 = 0.0f, p3 = 0.0f;
+    auto fetch = [&](int64_t span, int b) {
+        const bool ok = live && span < n_spans;
+        if (ok && r == 0) {
 #pragma unroll
-            for (int k = 0; k < 4; ++k) {
-                const float loc = xv[k] - av[k];
-                const float glob = mb[k] - av[k];
-                p0 = fmaf(loc, loc, p0);
-                p1 = fmaf(loc, glob, p1);
-                p2 = fmaf(glob, glob, p2);
-                p3 = fmaf(av[k], av[k], p3);
+            for (int j = 0; j < NV; ++j)
+                cp_async16(tiles + (b * R + M) * S + 4 * f + 4 * P * j, anchor + span * S + 4 * f + 4 * P * j);
+        }
+        fetch_row(ok, tiles + (b * R + r) * S + 4 * f, x + r * n + span * S + 4 * f, P);
+    };
+    fetch(blockIdx.x, 0);
+    int buf = 0;
+    for (int64_t span = blockIdx.x; span < n_spans; span += gridDim.x, buf ^= 1) {
+        fetch(span + gridDim.x, buf ^ 1);
+        cp_async_wait<1>();
+        __syncthreads();
+        const float *tile = tiles + buf * R * S;
+        const float *anc = tile + M * S;
+        tile_means(tile, M, log2_s, S, mean);
+        __syncthreads();
+        if (live) {
+            float p0 = 0.0f, p1 = 0.0f, p2 = 0.0f, p3 = 0.0f;   // this thread's 4 * NV elements
+#pragma unroll
+            for (int j = 0; j < NV; ++j) {
+                const int c = 4 * f + 4 * P * j;
+                float xv[4], mb[4], aj[4];
+                to_array(*reinterpret_cast<const float4 *>(tile + r * S + c), xv);
+                to_array(*reinterpret_cast<const float4 *>(mean + c), mb);
+                to_array(*reinterpret_cast<const float4 *>(anc + c), aj);
+#pragma unroll
+                for (int k = 0; k < 4; ++k) {
+                    const float loc = xv[k] - aj[k];
+                    const float glob = mb[k] - aj[k];
+                    p0 = fmaf(loc, loc, p0);
+                    p1 = fmaf(loc, glob, p1);
+                    p2 = fmaf(glob, glob, p2);
+                    p3 = fmaf(aj[k], aj[k], p3);
+                }
             }
             loc2.add(p0);
             cross.add(p1);
@@ -185,6 +234,7 @@ __global__ void __launch_bounds__(kWideMaxThreads) pseudo_grad_stats_wide_kernel
         }
         __syncthreads();
     }
+    cp_async_wait<0>();
 
     const double l2 = replica_lanes_sum(loc2.value(), P);
     const double c2 = replica_lanes_sum(cross.value(), P);
@@ -221,15 +271,16 @@ struct WideShape {
     size_t smem;
 };
 
-WideShape wide_shape(int M, int extra_floats) {
+WideShape wide_shape(int M, int extra_rows) {
     WideShape w;
     const int P = wide_positions(M);
     w.log2_p = 0;
     while ((1 << w.log2_p) < P) ++w.log2_p;
-    w.S = 4 * P;
+    w.S = 4 * P * kStatsVec;
     w.threads = (M * P + 31) / 32 * 32;
-    // the tile and the extra per-span vectors; the final reduction reuses it
-    size_t floats = static_cast<size_t>(M) * w.S + extra_floats * w.S;
+    // two tiles of M (+ extra) rows and the span's means; the final
+    // reduction reuses the tiles
+    const size_t floats = 2 * static_cast<size_t>(M + extra_rows) * w.S + w.S;
     const size_t red = 2 * (3 * static_cast<size_t>(M) + 2);   // doubles -> floats
     w.smem = (floats > red ? floats : red) * sizeof(float);
     return w;
@@ -268,15 +319,15 @@ cudaError_t launch_sync_stats_wide(const SyncArgs &a, int num_sms, double *parti
     if (a.n_sel <= 0) return cudaSuccess;
     if (a.M < 2 || a.M > kWideMaxM) return cudaErrorNotSupported;
     const int Q = 2 + 2 * a.M;
-    const WideShape w = wide_shape(a.M, 1);
-    const int per_sm = wide_blocks_per_sm(sync_stats_wide_kernel, w);
-    if (static_cast<size_t>(Q) * a.n_sel > partial_cap) return cudaErrorInvalidValue;
-    const int g = wide_grid(per_sm, num_sms, a.n_sel, a.n_padded / w.S, Q, partial_cap);
-    if (w.smem > 48 * 1024) {
+    const WideShape w = wide_shape(a.M, 0);
+    if (w.smem > 48 * 1024) {        // before the occupancy query, which depends on it
         cudaError_t e = cudaFuncSetAttribute(sync_stats_wide_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                              static_cast<int>(w.smem));
         if (e != cudaSuccess) return e;
     }
+    const int per_sm = wide_blocks_per_sm(sync_stats_wide_kernel, w);
+    if (static_cast<size_t>(Q) * a.n_sel > partial_cap) return cudaErrorInvalidValue;
+    const int g = wide_grid(per_sm, num_sms, a.n_sel, a.n_padded / w.S, Q, partial_cap);
     sync_stats_wide_kernel<<<dim3(g, a.n_sel), w.threads, w.smem, stream>>>(a, w.log2_p, partial);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
@@ -289,15 +340,15 @@ cudaError_t launch_pseudo_grad_stats_wide(const float *x, const float *anchor, i
                                           cudaStream_t stream) {
     if (M < 2 || M > kWideMaxM) return cudaErrorNotSupported;
     const int Q = 2 * M + 2;
-    const WideShape w = wide_shape(M, 2);
-    const int per_sm = wide_blocks_per_sm(pseudo_grad_stats_wide_kernel, w);
-    if (static_cast<size_t>(Q) > partial_cap) return cudaErrorInvalidValue;
-    const int g = wide_grid(per_sm, num_sms, 1, n / w.S, Q, partial_cap);
-    if (w.smem > 48 * 1024) {
+    const WideShape w = wide_shape(M, 1);
+    if (w.smem > 48 * 1024) {        // before the occupancy query, which depends on it
         cudaError_t e = cudaFuncSetAttribute(pseudo_grad_stats_wide_kernel,
                                              cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(w.smem));
         if (e != cudaSuccess) return e;
     }
+    const int per_sm = wide_blocks_per_sm(pseudo_grad_stats_wide_kernel, w);
+    if (static_cast<size_t>(Q) > partial_cap) return cudaErrorInvalidValue;
+    const int g = wide_grid(per_sm, num_sms, 1, n / w.S, Q, partial_cap);
     pseudo_grad_stats_wide_kernel<<<g, w.threads, w.smem, stream>>>(x, anchor, n, M, w.log2_p, partial);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;

@@ -1,8 +1,8 @@
 // step_sync_kernels.cuh -- the local step with the replica average fused in.
 //
 // step_sync_kernel is element-major: a lane updates the same few elements
-// of all M replicas (M <= 7) or of a share of them while other lanes of the
-// warp hold the rest (M = 8 and 16; see FusedShape), with the update of
+// of all M replicas (M <= 7) or of half of them while the other half-warp
+// holds the rest (M = 8; see FusedShape), with the update of
 // step_kernels.cuh; then it writes each state due for averaging as the
 // replica mean (E_m[.] of Algorithms 1-3) instead of the local values.  The
 // average costs no HBM traffic beyond the step's own.
@@ -23,14 +23,14 @@ namespace mtdao {
 //   M = 5, 6, 7 : one group, R = M, V = 2 (four elements spill registers);
 //   M = 8       : two groups (half-warps) of R = 4, V = 4: replicas 0..3 and
 //                 4..7 are the two parts of the compensated mean of
-//                 replica_mean.cuh, combined by shuffles;
-//   M = 16      : four groups of R = 4, V = 4; each part of the mean spans
-//                 two groups and its compensated sum is handed from one to
-//                 the next in replica order.
-// Other M up to 64 take the block-staged kernel of step_sync_wide.cuh (a
-// lane-group shape for M = 32, eight groups of four lanes, loaded 64-byte
-// pieces of eight replica slabs and ran slower than the separate average);
-// above 64, the plain step followed by the standalone average.
+//                 replica_mean.cuh, combined by shuffles.
+// M from 9 to 64 take the block-staged kernel of step_sync_wide.cuh (lane
+// groups went further before: M = 16 as four groups of four replicas, the
+// compensated sums handed from group to group by shuffles, ran at 4.9-5.3
+// TB/s against 5.2 for the block-staged kernel with every state due and 5.7
+// against 6.8 with x alone; M = 32 as eight groups loaded 64-byte pieces of
+// eight replica slabs and ran slower than the separate average); above 64,
+// the plain step followed by the standalone average.
 // The states are visited one after another (state_order); the next
 // state's loads are issued before the current state is updated and stored,
 // so two states' loads are in flight per lane within the 128-register cap.
@@ -42,8 +42,8 @@ namespace mtdao {
 // step_kernel) to 6582-6718; M = 2 is the same with or without it.
 template <int M>
 struct FusedShape {
-    static_assert((M >= 2 && M <= 8) || M == 16, "no fused shape for this M");
-    static constexpr int G = M == 16 ? 4 : M == 8 ? 2 : 1;    // lane groups per warp
+    static_assert(M >= 2 && M <= 8, "no fused shape for this M");
+    static constexpr int G = M == 8 ? 2 : 1;                  // lane groups per warp
     static constexpr int R = M / G;                          // replicas per lane
     static constexpr int V = (M >= 5 && M <= 7) ? 2 : 4;     // elements per lane
     static constexpr int kLanes = 32 / G;                    // lanes per group
@@ -104,44 +104,6 @@ __device__ __forceinline__ void store_replicas(float *state, int64_t n_padded, i
         for (int k = 0; k < S::V; ++k) {
             if constexpr (S::G == 1) {
                 mean[k] = replica_mean<M>([&](int m) { return val[m][k]; });
-            } else if constexpr (S::G >= 4) {
-                // Each part spans G/2 consecutive groups: its compensated sum
-                // is continued group by group in replica order (the running
-                // sum and compensation handed on by shuffles), then both
-                // parts are read from their last groups.
-                constexpr int H = S::G / 2;
-                const int pos = grp % H;
-                const int q = threadIdx.x & (S::kLanes - 1);
-                const float s0 = __shfl_sync(0xffffffffu, val[0][k], q);
-                DiffSum part(s0);
-#pragma unroll
-                for (int j = 0; j < H; ++j) {
-                    if (pos == j) {
-#pragma unroll
-                        for (int r = 0; r < S::R; ++r)
-                            if (r > 0 || grp != 0) part.add(val[r][k]);
-                    }
-                    if (j + 1 < H) {
-                        const float ps = __shfl_up_sync(0xffffffffu, part.sum, S::kLanes);
-                        const float pc = __shfl_up_sync(0xffffffffu, part.comp, S::kLanes);
-                        if (pos == j + 1) {
-                            part.sum = ps;
-                            part.comp = pc;
-                        }
-                    }
-                }
-                const float fin = part.partial();
-                const float a = __shfl_sync(0xffffffffu, fin, (H - 1) * S::kLanes + q);      // replicas 1 .. M/2-1
-                const float b = __shfl_sync(0xffffffffu, fin, (S::G - 1) * S::kLanes + q);   // replicas M/2 .. M-1
-                // plain sum for the non-finite case: every group's lanes end with
-                // the same bits (a + b == b + a)
-                float plain = val[0][k];
-#pragma unroll
-                for (int r = 1; r < S::R; ++r) plain += val[r][k];
-#pragma unroll
-                for (int off = S::kLanes; off < 32; off <<= 1) plain += __shfl_xor_sync(0xffffffffu, plain, off);
-                mean[k] = mean_or_plain(replica_mean_from_parts(s0, a, b, static_cast<float>(M)), plain,
-                                        static_cast<float>(M));
             } else {
                 // replica 0 lives in group 0: its value is the reference of both parts
                 const float s0 = __shfl_sync(0xffffffffu, val[0][k], threadIdx.x & (S::kLanes - 1));
@@ -324,7 +286,6 @@ cudaError_t launch_step_sync_m(const StepArgs &a, int num_sms, cudaStream_t st) 
         case 6: return launch_step_sync_t<BASE, N, GDT, CLIP, 6>(a, num_sms, st);
         case 7: return launch_step_sync_t<BASE, N, GDT, CLIP, 7>(a, num_sms, st);
         case 8: return launch_step_sync_t<BASE, N, GDT, CLIP, 8>(a, num_sms, st);
-        case 16: return launch_step_sync_t<BASE, N, GDT, CLIP, 16>(a, num_sms, st);
         default: return launch_step_sync_wide<BASE, N, GDT, CLIP>(a, st);
     }
 }

@@ -30,6 +30,7 @@ constexpr int kWideMaxM = 256;            // largest M of the span layout (diagn
 constexpr int kWideFusedMaxM = 64;        // largest M of the fused step (above: step + average)
 constexpr int kWideMaxThreads = 512;      // largest block of the span layout
 constexpr int kWideVec = 1;               // float4 positions per thread and state in the fused step
+constexpr int kWideVecLog2 = kWideVec == 1 ? 0 : kWideVec == 2 ? 1 : 2;
 
 // Threads per replica row of the span (a power of two).
 constexpr int wide_positions(int M) { return M <= 16 ? 16 : M <= 64 ? 8 : M <= 128 ? 4 : 2; }
@@ -40,33 +41,36 @@ constexpr int wide_span(int M) { return 4 * kWideVec * wide_positions(M); }
 constexpr int wide_floats_per_state(int M) { return (M + 1) * wide_span(M); }
 
 // Replica means of the n_cols columns of a block's tile into mean[p]
-// (column p: tile + (p / S) * M * S + p % S, the replicas at stride S).
+// (column p: tile + (p / S) * M * S + p % S, the replicas at stride
+// S = 2^log2_s; shifts, not a division by a run-time S).
 // Lanes 2i and 2i + 1 form the two compensated parts of replica_mean.cuh
 // for one column, replicas 1 .. h-1 and h .. M-1 in order (h = M / 2), and
 // join them with a shuffle: the bits of replica_mean_rt (with its plain
 // mean where the compensated one is NaN).  Every thread of
 // the block calls it (the shuffles take whole warps: blockDim.x is a
 // multiple of 32 and the loop count is the same for all threads).
-__device__ __forceinline__ void tile_means(const float *tile, int M, int S, int n_cols, float *mean) {
+__device__ __forceinline__ void tile_means(const float *tile, int M, int log2_s, int n_cols, float *mean) {
     const int t = threadIdx.x;
     const int h = M / 2;
+    const int S = 1 << log2_s;
     for (int p0 = 0; p0 < n_cols; p0 += static_cast<int>(blockDim.x >> 1)) {
         const int p = p0 + (t >> 1);
         const int part = t & 1;
         float s0 = 0.0f, mine = 0.0f;
         if (p < n_cols) {
-            const float *col = tile + (p / S) * M * S + (p & (S - 1));
+            const float *col = tile + (p >> log2_s) * M * S + (p & (S - 1));
             s0 = col[0];
             DiffSum sum(s0);
             const int lo = part ? h : 1, hi = part ? M : h;
-            for (int m = lo; m < hi; ++m) sum.add(col[m * S]);
+#pragma unroll 4
+            for (int m = lo; m < hi; ++m) sum.add(col[m * S]);   // unrolled: the loads run ahead
             mine = sum.partial();
         }
         const float other = __shfl_xor_sync(0xffffffffu, mine, 1);
         if (p < n_cols && part == 0) {
             float v = replica_mean_from_parts(s0, mine, other, static_cast<float>(M));
             if (v != v) {                        // non-finite values: the plain mean (replica_mean.cuh)
-                const float *col = tile + (p / S) * M * S + (p & (S - 1));
+                const float *col = tile + (p >> log2_s) * M * S + (p & (S - 1));
                 float plain = col[0];
                 for (int m = 1; m < M; ++m) plain += col[m * S];
                 v = plain / static_cast<float>(M);
@@ -131,7 +135,7 @@ __global__ void __launch_bounds__(kWideMaxThreads) step_sync_wide_kernel(const S
             }
         }
         __syncthreads();
-        tile_means(tile, M, S, n_due * S, mean);
+        tile_means(tile, M, log2_p + 2 + kWideVecLog2, n_due * S, mean);
         __syncthreads();
         if (live) {
 #pragma unroll
