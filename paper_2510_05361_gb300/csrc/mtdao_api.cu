@@ -527,7 +527,7 @@ static int ensure_stats_workspace(mtdao_ctx *h) {
     if (h->stats_partial == nullptr) {
         const size_t cap = path == kStatsGeneral ? general_stats_partial_capacity(h->num_sms, h->M)
                            : path == kStatsWide  ? wide_stats_partial_capacity(h->num_sms, h->n_states, h->M)
-                                                 : sync_stats_partial_capacity(h->num_sms, h->n_states, h->M);
+                                                 : sync_stats_partial_capacity(h->num_sms, h->n_padded, h->n_states, h->M);
         cudaError_t e = cudaMalloc(reinterpret_cast<void **>(&h->stats_partial), cap * sizeof(double));
         if (e != cudaSuccess) {
             cudaGetLastError();

@@ -80,7 +80,7 @@ cudaError_t launch_sync(const SyncArgs &a, int num_sms, cudaStream_t stream);
 // stats[sel * (2 + 2M) + q], q as documented for mtdao_sync_stats.  Needs a
 // workspace of sync_stats_partial_capacity() doubles; M must be 1..8
 // (cudaErrorNotSupported otherwise).
-size_t sync_stats_partial_capacity(int num_sms, int n_states, int M);
+size_t sync_stats_partial_capacity(int num_sms, int64_t n_padded, int n_states, int M);
 cudaError_t launch_sync_stats(const SyncArgs &a, int num_sms, double *partial, size_t partial_cap,
                               double *stats, cudaStream_t stream);
 

@@ -233,13 +233,28 @@ __global__ void __launch_bounds__(kNormThreads) sqnorm_finalize_kernel(const dou
 
 // ---------------------------------------------------------------- sync + diagnostics
 
+// Float4 positions a thread of sync_stats_kernel takes, consecutive for its
+// block: block b covers positions [b * tile * 256, (b + 1) * tile * 256).
+// One block per tile, started in index order as earlier blocks retire;
+// every block leaves one row of sums for stats_finalize_kernel, so the sums
+// do not depend on the SM count.  A block's fixed cost is that row (2M + 2
+// warp and block reductions in fp64), so the tile must be long.  On the ~1B
+// and ~350M workloads this launch took the sync with diagnostics from
+// 6426 / 6335 GB/s (persistent grid: occupancy x SMs blocks, grid-stride)
+// to 6712 / 6696.  On flat 2^30-element sets (GB/s at M = 4 / 8):
+// persistent 5943 / 6139; tiles of 2: 1621 / 1795, 8: 5638 / 4590,
+// 32: 6152 / 6275, 128: 6121 / 6308, 512: 6051 / 6173.  The read-only
+// pseudo-gradient pass keeps the persistent grid: with tiles of 512 it ran
+// 6212 / 5908 GB/s on the two workloads against 7153 / 6237.
+constexpr int kSyncStatsTile = 128;
+
 // Replica average of the selected states (exactly as sync_kernel) plus, in
 // the same pass over the M replicas, per state and block the partial sums of
 //   q = 0          sum_m (s_m - s_bar)^2        (cross-worker variance * M)
 //   q = 1          s_bar^2
 //   q = 2 + m      s_m^2
 //   q = 2 + M + m  s_m * s_bar
-// written to partial[(sel * gridDim.x + block) * Q + q], Q = 2 + 2M.  s_bar
+// written to partial[(sel * Q + q) * gridDim.x + block], Q = 2 + 2M.  s_bar
 // is the fp32 mean that is stored.  With M = 1 nothing is stored (there is
 // nothing to average) but the sums are still formed.
 template <int M>
@@ -249,8 +264,10 @@ __global__ void __launch_bounds__(kThreads) sync_stats_kernel(const SyncArgs a, 
     const int64_t n = a.n_padded;
     const int64_t nv = n / 4;
     Kahan acc[Q];
-    for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < nv;
-         i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+    const int64_t first = static_cast<int64_t>(blockIdx.x) * kSyncStatsTile * blockDim.x + threadIdx.x;
+    for (int k = 0; k < kSyncStatsTile; ++k) {
+        const int64_t i = first + static_cast<int64_t>(k) * blockDim.x;
+        if (i >= nv) break;
         const int64_t e = 4 * i;
         float r[M][4];
 #pragma unroll
@@ -291,44 +308,53 @@ __global__ void __launch_bounds__(kThreads) sync_stats_kernel(const SyncArgs a, 
     if (threadIdx.x < Q) {
         double total = 0.0;
         for (int i = 0; i < static_cast<int>(blockDim.x >> 5); ++i) total += part[threadIdx.x][i];
-        partial[(static_cast<int64_t>(blockIdx.y) * gridDim.x + blockIdx.x) * Q + threadIdx.x] = total;
+        partial[(static_cast<int64_t>(blockIdx.y) * Q + threadIdx.x) * gridDim.x + blockIdx.x] = total;
     }
 }
 
-// stats[sel * Q + q] = sum over blocks of partial (in block order); q = 0 is
-// divided by divide_first (M for the variance, a mean over workers)
-// (divide_first = 0 leaves q = 0 undivided)
-__global__ void sync_stats_finalize_kernel(const double *partial, int blocks, int Q, int divide_first,
-                                           double *stats) {
-    const int sel = blockIdx.x, q = threadIdx.x;
-    if (q >= Q) return;
-    double total = 0.0;
-    for (int b = 0; b < blocks; ++b) total += partial[(static_cast<int64_t>(sel) * blocks + b) * Q + q];
-    stats[sel * Q + q] = (q == 0 && divide_first > 0) ? total / divide_first : total;
+// stats[row * Q + q] = the sum over blocks of partial[(row * Q + q) * blocks + b]:
+// thread t of block (q, row) adds a contiguous run of blocks in order, then
+// block_sum adds the threads' sums in a fixed order.  q = 0 is divided by
+// divide_first (M for the variance, a mean over workers; 0 leaves it).
+__global__ void __launch_bounds__(kNormThreads) stats_finalize_kernel(const double *partial, int64_t blocks,
+                                                                      int Q, int divide_first, double *stats) {
+    const int q = blockIdx.x, row = blockIdx.y;
+    const double *p = partial + (static_cast<int64_t>(row) * Q + q) * blocks;
+    const int64_t per = (blocks + blockDim.x - 1) / blockDim.x;
+    const int64_t lo = threadIdx.x * per;
+    const int64_t hi = lo + per < blocks ? lo + per : blocks;
+    double acc = 0.0;
+    for (int64_t b = lo; b < hi; ++b) acc += p[b];
+    const double total = block_sum(acc);
+    if (threadIdx.x == 0) stats[row * Q + q] = (q == 0 && divide_first > 0) ? total / divide_first : total;
+}
+
+// Blocks of a register-resident diagnostics kernel per state: each covers
+// `tile` consecutive float4 positions per thread.
+int64_t stats_blocks(int64_t n_padded, int tile) {
+    const int64_t nv = n_padded / 4;
+    const int64_t per_block = static_cast<int64_t>(tile) * kThreads;
+    const int64_t b = (nv + per_block - 1) / per_block;
+    return b < 1 ? 1 : b;
 }
 
 template <int M>
-cudaError_t launch_sync_stats_t(const SyncArgs &a, int num_sms, double *partial, size_t partial_cap,
-                                double *stats, cudaStream_t stream) {
+cudaError_t launch_sync_stats_t(const SyncArgs &a, double *partial, size_t partial_cap, double *stats,
+                                cudaStream_t stream) {
     constexpr int Q = 2 + 2 * M;
-    static const int per_sm = blocks_per_sm(sync_stats_kernel<M>);
-    const int64_t nv = a.n_padded / 4;
-    int64_t gx = static_cast<int64_t>(per_sm) * num_sms / a.n_sel;
-    const int64_t need = (nv + kThreads - 1) / kThreads;
-    if (gx > need) gx = need;
-    if (gx < 1) gx = 1;
-    if (static_cast<size_t>(gx) * a.n_sel * Q > partial_cap) return cudaErrorInvalidValue;
+    const int64_t gx = stats_blocks(a.n_padded, kSyncStatsTile);
+    if (static_cast<size_t>(gx) * a.n_sel * Q > partial_cap || gx > 0x7fffffff) return cudaErrorInvalidValue;
     dim3 grid(static_cast<unsigned>(gx), static_cast<unsigned>(a.n_sel));
     sync_stats_kernel<M><<<grid, kThreads, 0, stream>>>(a, partial);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
-    sync_stats_finalize_kernel<<<a.n_sel, 32, 0, stream>>>(partial, static_cast<int>(gx), Q, M, stats);
+    stats_finalize_kernel<<<dim3(Q, a.n_sel), kNormThreads, 0, stream>>>(partial, gx, Q, M, stats);
     return cudaGetLastError();
 }
 
 // Pseudo-gradient diagnostics of the parameters x[M][n] against the anchor
-// a[n] (the parameters at the last average), read-only, with fixed-order
-// sums into partial[block * Q + q], Q = 2M + 2:
+// a[n] (the parameters at the last average), read-only, on a persistent
+// grid, with fixed-order sums into partial[q * gridDim.x + block], Q = 2M + 2:
 //   q = m          (x_m - a)^2
 //   q = M + m      (x_m - a) * (x_bar - a)
 //   q = 2M         (x_bar - a)^2
@@ -378,7 +404,7 @@ __global__ void __launch_bounds__(kThreads) pseudo_grad_stats_kernel(const float
     if (threadIdx.x < Q) {
         double total = 0.0;
         for (int i = 0; i < static_cast<int>(blockDim.x >> 5); ++i) total += part[threadIdx.x][i];
-        partial[static_cast<int64_t>(blockIdx.x) * Q + threadIdx.x] = total;
+        partial[static_cast<int64_t>(threadIdx.x) * gridDim.x + blockIdx.x] = total;
     }
 }
 
@@ -396,11 +422,10 @@ cudaError_t launch_pseudo_grad_stats_t(const float *x, const float *anchor, int6
     pseudo_grad_stats_kernel<M><<<static_cast<unsigned>(gx), kThreads, 0, stream>>>(x, anchor, n, partial);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
-    // same fixed-order finalisation as the sync diagnostics, with no division
-    sync_stats_finalize_kernel<<<1, 32, 0, stream>>>(partial, static_cast<int>(gx), Q, 0, stats);
+    // the same fixed-order finalisation as the sync diagnostics, with no division
+    stats_finalize_kernel<<<dim3(Q, 1), kNormThreads, 0, stream>>>(partial, gx, Q, 0, stats);
     return cudaGetLastError();
 }
-
 
 // ---------------------------------------------------------------- diagnostics for any M
 
@@ -677,23 +702,26 @@ cudaError_t launch_pseudo_grad_stats(const float *x, const float *anchor, int64_
     }
 }
 
-size_t sync_stats_partial_capacity(int num_sms, int n_states, int M) {
-    // at most 16 resident blocks per SM of 256 threads, split over the states
-    return static_cast<size_t>(16 * num_sms + n_states) * (2 + 2 * M);
+size_t sync_stats_partial_capacity(int num_sms, int64_t n_padded, int n_states, int M) {
+    // one row of 2 + 2M sums per block and state, or per persistent block
+    // of the pseudo-gradient pass (at most 16 resident blocks per SM)
+    const size_t sync = static_cast<size_t>(stats_blocks(n_padded, kSyncStatsTile)) * n_states;
+    const size_t change = static_cast<size_t>(16) * num_sms;
+    return (sync > change ? sync : change) * (2 + 2 * static_cast<size_t>(M));
 }
 
 cudaError_t launch_sync_stats(const SyncArgs &a, int num_sms, double *partial, size_t partial_cap,
                               double *stats, cudaStream_t stream) {
     if (a.n_sel <= 0) return cudaSuccess;
     switch (a.M) {
-        case 1: return launch_sync_stats_t<1>(a, num_sms, partial, partial_cap, stats, stream);
-        case 2: return launch_sync_stats_t<2>(a, num_sms, partial, partial_cap, stats, stream);
-        case 3: return launch_sync_stats_t<3>(a, num_sms, partial, partial_cap, stats, stream);
-        case 4: return launch_sync_stats_t<4>(a, num_sms, partial, partial_cap, stats, stream);
-        case 5: return launch_sync_stats_t<5>(a, num_sms, partial, partial_cap, stats, stream);
-        case 6: return launch_sync_stats_t<6>(a, num_sms, partial, partial_cap, stats, stream);
-        case 7: return launch_sync_stats_t<7>(a, num_sms, partial, partial_cap, stats, stream);
-        case 8: return launch_sync_stats_t<8>(a, num_sms, partial, partial_cap, stats, stream);
+        case 1: return launch_sync_stats_t<1>(a, partial, partial_cap, stats, stream);
+        case 2: return launch_sync_stats_t<2>(a, partial, partial_cap, stats, stream);
+        case 3: return launch_sync_stats_t<3>(a, partial, partial_cap, stats, stream);
+        case 4: return launch_sync_stats_t<4>(a, partial, partial_cap, stats, stream);
+        case 5: return launch_sync_stats_t<5>(a, partial, partial_cap, stats, stream);
+        case 6: return launch_sync_stats_t<6>(a, partial, partial_cap, stats, stream);
+        case 7: return launch_sync_stats_t<7>(a, partial, partial_cap, stats, stream);
+        case 8: return launch_sync_stats_t<8>(a, partial, partial_cap, stats, stream);
         default: return cudaErrorNotSupported;
     }
 }
