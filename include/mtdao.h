@@ -357,9 +357,10 @@ int mtdao_sync_due(mtdao_handle h, uint32_t *mask_out);
  * doubles, caller-owned, 8-byte aligned) receives sum_i g[m][i]^2.
  * Deterministic: fixed grid and fixed reduction order.  Squares are summed
  * in fp32 with compensation where they stay within fp32's range; groups of
- * four values whose squares overflow or underflow fp32 (|g| above ~1e19 or
- * below ~1e-19) are summed in fp64, so every finite gradient gives a finite,
- * accurate sum.  Uses a handle-owned workspace of partial sums.
+ * four f32 or eight bf16 values (one 16-byte load) whose squares overflow or
+ * underflow fp32 (|g| above ~1e19 or below ~1e-19) are summed in fp64, so
+ * every finite gradient gives a finite, accurate sum.  Uses a handle-owned
+ * workspace of partial sums.
  * Errors: MTDAO_ERR_INVALID, MTDAO_ERR_ALIGN, MTDAO_ERR_CUDA.
  */
 int mtdao_grad_sqnorm(mtdao_handle h, const void *grads_dev, int32_t grad_dtype,

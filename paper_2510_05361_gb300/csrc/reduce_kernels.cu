@@ -106,34 +106,49 @@ __device__ double block_sum(double v) {
     return total;
 }
 
-// Positions (groups of 4 elements) a thread of the norm kernels loads
-// before it accumulates them: i, i + T, ..., i + (U - 1) T with T the
-// replica's thread count, the same order as a plain grid-stride loop, so
-// the sums do not depend on the unrolling.  64 bytes per thread in flight:
-// 4 positions of f32, 8 of bf16.
-template <int GDT>
-constexpr int kNormUnroll = GDT == MTDAO_F32 ? 4 : 8;
-
-// Four gradient values as loaded (f32: float4; bf16: two packed words, 2
-// registers instead of 4 until they are widened) and their fp32 values.
-template <int GDT>
-using GradWords = typename std::conditional<GDT == MTDAO_F32, float4, uint2>::type;
+// A position of the norm kernels is one 16-byte load of the gradient: 4 f32
+// or 8 bf16 values (8-byte bf16 loads, half the bytes per load instruction,
+// read the ~350M workload's gradients at 5.56 TB/s).  A thread loads
+// kNormUnroll positions before it accumulates them: i, i + T, ...,
+// i + (U - 1) T with T the replica's thread count, the same order as a
+// plain grid-stride loop, so the sums do not depend on the unrolling.
+// 64 bytes per thread in flight.
+constexpr int kNormUnroll = 4;
 
 template <int GDT>
-__device__ __forceinline__ GradWords<GDT> ld_grad_words(const void *g, int64_t e) {
+struct NormPos;
+template <>
+struct NormPos<MTDAO_F32> {
+    static constexpr int E = 4;
+    using W = float4;
+};
+template <>
+struct NormPos<MTDAO_BF16> {
+    static constexpr int E = 8;
+    using W = uint4;
+};
+
+template <int GDT>
+__device__ __forceinline__ typename NormPos<GDT>::W ld_grad_words(const void *g, int64_t e) {
     if constexpr (GDT == MTDAO_F32)
         return __ldcs(reinterpret_cast<const float4 *>(static_cast<const float *>(g) + e));
     else
-        return __ldcs(reinterpret_cast<const uint2 *>(static_cast<const uint16_t *>(g) + e));
+        return __ldcs(reinterpret_cast<const uint4 *>(static_cast<const uint16_t *>(g) + e));
 }
 
+// The position's values in fp32 (bf16 -> fp32 is exact: the bits move up by 16).
 template <int GDT>
-__device__ __forceinline__ float4 widen(GradWords<GDT> w) {
-    if constexpr (GDT == MTDAO_F32)
-        return w;
-    else
-        return make_float4(__uint_as_float(w.x << 16), __uint_as_float(w.x & 0xffff0000u),
-                           __uint_as_float(w.y << 16), __uint_as_float(w.y & 0xffff0000u));
+__device__ __forceinline__ void widen(const typename NormPos<GDT>::W &w, float (&q)[NormPos<GDT>::E]) {
+    if constexpr (GDT == MTDAO_F32) {
+        q[0] = w.x; q[1] = w.y; q[2] = w.z; q[3] = w.w;
+    } else {
+        const uint32_t u[4] = {w.x, w.y, w.z, w.w};
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+            q[2 * k] = __uint_as_float(u[k] << 16);
+            q[2 * k + 1] = __uint_as_float(u[k] & 0xffff0000u);
+        }
+    }
 }
 
 // fp32 range of a position's sum of four squares that the Kahan sum takes:
@@ -151,28 +166,37 @@ constexpr float kSqLo = 0x1p-100f;
 template <int GDT>
 __global__ void __launch_bounds__(kNormThreads, 4) sqnorm_partial_kernel(const void *g, int64_t n,
                                                                       double *partial) {
+    constexpr int E = NormPos<GDT>::E;
     const int m = blockIdx.y;
     const int nb = gridDim.x;
-    const int64_t nv = n / 4;
+    const int64_t np = n / E;
     const int64_t T = static_cast<int64_t>(nb) * blockDim.x;
     float sum = 0.0f, comp = 0.0f;
     double wide = 0.0;                 // positions outside [kSqLo, kSqHi]
-    for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < nv;
-         i += kNormUnroll<GDT> * T) {
-        GradWords<GDT> w[kNormUnroll<GDT>];
+    for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < np;
+         i += kNormUnroll * T) {
+        typename NormPos<GDT>::W w[kNormUnroll];
 #pragma unroll
-        for (int u = 0; u < kNormUnroll<GDT>; ++u)
-            if (i + u * T < nv) w[u] = ld_grad_words<GDT>(g, m * n + 4 * (i + u * T));
+        for (int u = 0; u < kNormUnroll; ++u)
+            if (i + u * T < np) w[u] = ld_grad_words<GDT>(g, m * n + E * (i + u * T));
 #pragma unroll
-        for (int u = 0; u < kNormUnroll<GDT>; ++u) {
-            if (i + u * T >= nv) break;
-            const float4 q = widen<GDT>(w[u]);
-            const float p = fmaf(q.x, q.x, fmaf(q.y, q.y, fmaf(q.z, q.z, __fmul_rn(q.w, q.w))));
-            const bool tiny = p < kSqLo && ((__float_as_uint(q.x) | __float_as_uint(q.y) | __float_as_uint(q.z) |
-                                             __float_as_uint(q.w)) & 0x7fffffffu) != 0u;
+        for (int u = 0; u < kNormUnroll; ++u) {
+            if (i + u * T >= np) break;
+            float q[E];
+            widen<GDT>(w[u], q);
+            float p = __fmul_rn(q[E - 1], q[E - 1]);
+            uint32_t bits = __float_as_uint(q[E - 1]);
+#pragma unroll
+            for (int k = E - 2; k >= 0; --k) {
+                p = fmaf(q[k], q[k], p);
+                bits |= __float_as_uint(q[k]);
+            }
+            const bool tiny = p < kSqLo && (bits & 0x7fffffffu) != 0u;
             if (!(p <= kSqHi) || tiny) {
-                const double a = q.x, b = q.y, c = q.z, d = q.w;
-                wide += fma(a, a, fma(b, b, fma(c, c, d * d)));
+                double d = static_cast<double>(q[E - 1]) * q[E - 1];
+#pragma unroll
+                for (int k = E - 2; k >= 0; --k) d = fma(static_cast<double>(q[k]), static_cast<double>(q[k]), d);
+                wide += d;
                 continue;
             }
             const float y = p - comp;
@@ -191,24 +215,26 @@ __global__ void __launch_bounds__(kNormThreads, 4) sqnorm_partial_kernel(const v
 template <int GDT>
 __global__ void __launch_bounds__(kNormThreads, 4) nonfinite_partial_kernel(const void *g, int64_t n,
                                                                          double *partial) {
+    constexpr int E = NormPos<GDT>::E;
     const int m = blockIdx.y;
     const int nb = gridDim.x;
-    const int64_t nv = n / 4;
+    const int64_t np = n / E;
     const int64_t T = static_cast<int64_t>(nb) * blockDim.x;
-    const uint32_t e = 0x7f800000u;
-    uint32_t count = 0;                // at most 4 nv / T per thread
-    for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < nv;
-         i += kNormUnroll<GDT> * T) {
-        GradWords<GDT> w[kNormUnroll<GDT>];
+    const uint32_t ex = 0x7f800000u;
+    uint32_t count = 0;                // at most E np / T per thread
+    for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < np;
+         i += kNormUnroll * T) {
+        typename NormPos<GDT>::W w[kNormUnroll];
 #pragma unroll
-        for (int u = 0; u < kNormUnroll<GDT>; ++u)
-            if (i + u * T < nv) w[u] = ld_grad_words<GDT>(g, m * n + 4 * (i + u * T));
+        for (int u = 0; u < kNormUnroll; ++u)
+            if (i + u * T < np) w[u] = ld_grad_words<GDT>(g, m * n + E * (i + u * T));
 #pragma unroll
-        for (int u = 0; u < kNormUnroll<GDT>; ++u) {
-            if (i + u * T >= nv) break;
-            const float4 q = widen<GDT>(w[u]);
-            count += ((__float_as_uint(q.x) & e) == e) + ((__float_as_uint(q.y) & e) == e) +
-                     ((__float_as_uint(q.z) & e) == e) + ((__float_as_uint(q.w) & e) == e);
+        for (int u = 0; u < kNormUnroll; ++u) {
+            if (i + u * T >= np) break;
+            float q[E];
+            widen<GDT>(w[u], q);
+#pragma unroll
+            for (int k = 0; k < E; ++k) count += (__float_as_uint(q[k]) & ex) == ex;
         }
     }
     const double total = block_sum(static_cast<double>(count));
