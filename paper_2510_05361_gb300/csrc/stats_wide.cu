@@ -42,16 +42,6 @@ __device__ __forceinline__ double replica_lanes_sum(double v, int P) {
 constexpr int kStatsVec = 4;
 constexpr int kStatsVecLog2 = 2;
 
-// 16-byte asynchronous global -> shared copies (cp.async, L2 only) and their
-// groups: a block copies the next span's tile while it works on this one.
-__device__ __forceinline__ void cp_async16(float *smem_dst, const float *gmem_src) {
-    const unsigned dst = static_cast<unsigned>(__cvta_generic_to_shared(smem_dst));
-    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;\n" ::"r"(dst), "l"(gmem_src) : "memory");
-}
-__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::: "memory"); }
-template <int N>
-__device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;\n" ::"n"(N) : "memory"); }
-
 // Copies this thread's kStatsVec float4 positions of replica r of a span
 // (src: the replica's first element of the span) into its tile row, then
 // commits the group (an empty one when the span is past the end).

@@ -286,7 +286,7 @@ cudaError_t launch_step_sync_m(const StepArgs &a, int num_sms, cudaStream_t st) 
         case 6: return launch_step_sync_t<BASE, N, GDT, CLIP, 6>(a, num_sms, st);
         case 7: return launch_step_sync_t<BASE, N, GDT, CLIP, 7>(a, num_sms, st);
         case 8: return launch_step_sync_t<BASE, N, GDT, CLIP, 8>(a, num_sms, st);
-        default: return launch_step_sync_wide<BASE, N, GDT, CLIP>(a, st);
+        default: return launch_step_sync_wide<BASE, N, GDT, CLIP>(a, num_sms, st);
     }
 }
 

@@ -2,23 +2,28 @@
 // for replica counts from 9 to 64 (kWideFusedMaxM), and the span layout
 // that the one-pass diagnostics of stats_wide.cu share (up to kWideMaxM).
 //
-// A block owns a span of S consecutive elements of all M replicas.  Thread
-// (r, f) of the block updates kWideVec float4 positions of the span in
-// replica r (f, f + P, ...) with update_state, issuing every state's loads
-// before any arithmetic.  A state that is not due is stored at once.  A due
-// state goes to shared memory instead; after one barrier the replica mean
-// of every (due state, element) pair is formed by two threads, each running
-// one of the two compensated parts of replica_mean.cuh over the replicas in
-// order, joined by one shuffle; after a second barrier every thread stores
-// the means to its own replica.  The parts are the ones the standalone
-// average forms (sync_kernel's streamed loop), in the same order, so fused
-// and separate averaging give identical bits for every M.
+// A block owns a span of S consecutive elements of all M replicas; thread
+// (r, f) updates elements [4f, 4f + 4) of replica r (and [4(f + P), ...)
+// for M > 16, see wide_fused_vec) with update_state.  The
+// blocks are persistent and double-buffer their spans in shared memory: the
+// next span of every state and of the gradient is copied in with cp.async
+// while the current one is updated, so HBM traffic continues through the
+// barriers.  A state that is not due is stored from registers at once; a
+// due state's new values go back over its tile in shared memory; after one
+// barrier the replica mean of every (due state, element) pair is formed by
+// two threads, each running one of the two compensated parts of
+// replica_mean.cuh over the replicas in order, joined by one shuffle; after
+// a second barrier every thread stores the means to its own replica.  The
+// parts are the ones the standalone average forms (sync_kernel's streamed
+// loop), in the same order, so fused and separate averaging give identical
+// bits for every M.
 //
 // Rows of the span are 32 bytes or longer: P = 16 (M <= 16), 8 (M <= 64),
 // 4 (M <= 128), 2 (M <= 256) float4 positions per thread row, so a block
 // has M * P <= 512 threads (rounded up to whole warps; threads beyond M * P
-// only take part in the mean).  Shared memory: one M x S tile and S means
-// per due state.
+// only take part in the mean).  Shared memory of the fused step: two span
+// buffers (a tile per state and the gradient tile) and S means per due
+// state.
 #pragma once
 
 #include "replica_mean.cuh"
@@ -29,16 +34,10 @@ namespace mtdao {
 constexpr int kWideMaxM = 256;            // largest M of the span layout (diagnostics)
 constexpr int kWideFusedMaxM = 64;        // largest M of the fused step (above: step + average)
 constexpr int kWideMaxThreads = 512;      // largest block of the span layout
-constexpr int kWideVec = 1;               // float4 positions per thread and state in the fused step
-constexpr int kWideVecLog2 = kWideVec == 1 ? 0 : kWideVec == 2 ? 1 : 2;
 
 // Threads per replica row of the span (a power of two).
 constexpr int wide_positions(int M) { return M <= 16 ? 16 : M <= 64 ? 8 : M <= 128 ? 4 : 2; }
 
-// Elements of the fused step's span, and its floats of shared memory per
-// due state: the M x S tile and S means.
-constexpr int wide_span(int M) { return 4 * kWideVec * wide_positions(M); }
-constexpr int wide_floats_per_state(int M) { return (M + 1) * wide_span(M); }
 
 // Replica means of the n_cols columns of a block's tile into mean[p]
 // (column p: tile + (p / S) * M * S + p % S, the replicas at stride
@@ -80,14 +79,53 @@ __device__ __forceinline__ void tile_means(const float *tile, int M, int log2_s,
     }
 }
 
+// 16- and 8-byte asynchronous global -> shared copies (cp.async) and their
+// groups: a block copies its next span while it works on the current one.
+__device__ __forceinline__ void cp_async16(void *smem_dst, const void *gmem_src) {
+    const unsigned dst = static_cast<unsigned>(__cvta_generic_to_shared(smem_dst));
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;\n" ::"r"(dst), "l"(gmem_src) : "memory");
+}
+__device__ __forceinline__ void cp_async8(void *smem_dst, const void *gmem_src) {
+    const unsigned dst = static_cast<unsigned>(__cvta_generic_to_shared(smem_dst));
+    asm volatile("cp.async.ca.shared.global [%0], [%1], 8;\n" ::"r"(dst), "l"(gmem_src) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;\n" ::"n"(N) : "memory"); }
+
+// Floats of one span buffer: a tile of M x S floats per state and the
+// gradient tile (M x S f32, or bf16 in half the floats).
+template <int BASE, int N, int GDT>
+__host__ __device__ constexpr int wide_buffer_floats(int M, int S) {
+    return kNumStates<BASE, N> * M * S + (GDT == MTDAO_F32 ? M * S : M * S / 2);
+}
+
+// The fused step on spans of all replicas, persistent, double-buffered:
+// while a block updates span i from shared memory, span i + gridDim.x of
+// every state and of the gradient is on its way in (cp.async).  In a
+// buffer the due states' tiles come first (in state index order), so the
+// means read them as one [n_due][M][S] array; a due state's updated values
+// are written back over its own tile, a state that is not due goes
+// straight to HBM.
+// Float4 positions per thread and row of the fused step's span (the
+// positions f and f + P): rows of 256 bytes up to M = 32 (S = 64).  With one
+// position and P = 8 (rows of 128 bytes) M = 24 and 32 ran at 4.8-4.9 TB/s
+// (Adam, N = 3), with two at 5.4, against 5.7-6.0 for M = 12-16.
+// Above 32 two positions made a span buffer so large (up to 96 KB) that
+// one block fitted per SM: M = 48 and 64 fell from 4.9-5.0 to 3.9-4.2 TB/s.
+constexpr int wide_fused_vec(int M) { return (M > 16 && M <= 32) ? 2 : 1; }
+
 template <int BASE, int N, int GDT, bool CLIP>
-__global__ void __launch_bounds__(kWideMaxThreads) step_sync_wide_kernel(const StepArgs a, int log2_p) {
-    extern __shared__ float smem[];
+__global__ void __launch_bounds__(kWideMaxThreads) step_sync_wide_kernel(const StepArgs a, int log2_p,
+                                                                         int log2_v) {
+    extern __shared__ __align__(16) float smem[];
     constexpr int kStates = kNumStates<BASE, N>;
-    constexpr int NV = kWideVec;
+    constexpr int kMaxVec = 2;
     const int M = a.M;
     const int P = 1 << log2_p;
-    const int S = 4 * P * NV;                    // elements of the span
+    const int NV = 1 << log2_v;                  // float4 positions per thread (1 or 2)
+    const int log2_s = log2_p + 2 + log2_v;
+    const int S = 1 << log2_s;                   // elements of the span
     const int t = threadIdx.x;
     const int r = t >> log2_p;                   // replica of this thread
     const int f = t & (P - 1);                   // its first float4 position in the span
@@ -96,81 +134,128 @@ __global__ void __launch_bounds__(kWideMaxThreads) step_sync_wide_kernel(const S
     const int64_t n_spans = n / S;
     const uint32_t mask = a.sync_mask;
     const int n_due = __popc(mask);
-    float *tile = smem;                          // [n_due][M][S]
-    float *mean = smem + n_due * M * S;          // [n_due][S]
+    const int tile = M * S;
+    const int buf_floats = wide_buffer_floats<BASE, N, GDT>(M, S);
+    float *mean = smem + 2 * buf_floats;         // [n_due][S]
     const float s = (CLIP && live) ? __ldg(a.clip_scale + r) : 1.0f;
+    const int own = r * S + 4 * f;               // this thread's offset in a tile
+    // tile of state st in a buffer: the due states first
+    auto slot = [&](int st) {
+        const uint32_t below = (1u << st) - 1u;
+        return ((mask >> st) & 1u) ? __popc(mask & below) : n_due + __popc(~mask & below);
+    };
+    auto fetch = [&](int64_t span, float *buf) {
+        if (live && span < n_spans) {
+#pragma unroll
+            for (int j = 0; j < kMaxVec; ++j) {
+                if (j >= NV) break;
+                const int64_t src = r * n + span * S + 4 * f + 4 * P * j;
+                const int dst = own + 4 * P * j;
+#pragma unroll
+                for (int st = 0; st < kStates; ++st)
+                    cp_async16(buf + slot(st) * tile + dst, a.arena + st * a.stride + src);
+                if constexpr (GDT == MTDAO_F32)
+                    cp_async16(buf + kStates * tile + dst, static_cast<const float *>(a.grads) + src);
+                else
+                    cp_async8(reinterpret_cast<uint16_t *>(buf + kStates * tile) + dst,
+                              static_cast<const uint16_t *>(a.grads) + src);
+            }
+        }
+        cp_async_commit();
+    };
 
-    for (int64_t span = blockIdx.x; span < n_spans; span += gridDim.x) {
+    // one span ahead: span k of this block lives in buffer k % 2 (a third
+    // buffer, two spans ahead, measured the same or 5-10 % slower: fewer
+    // blocks fit per SM)
+    int b = 0;
+    fetch(blockIdx.x, smem);
+    for (int64_t span = blockIdx.x; span < n_spans; span += gridDim.x, b ^= 1) {
+        float *buf = smem + b * buf_floats;
+        fetch(span + gridDim.x, smem + (b ^ 1) * buf_floats);
+        cp_async_wait<1>();                      // this thread's copies of `span` have landed
+        __syncthreads();                         // ... and every thread's
         const int64_t e = span * S + 4 * f;      // element index within a replica (position j: + 4 P j)
         if (live) {
-            float g[NV][4], buf[kStates][NV][4], gt[NV][4], acc[NV][4];
 #pragma unroll
-            for (int j = 0; j < NV; ++j) to_array(ld_grad<GDT>(a.grads, r * n + e + 4 * P * j), g[j]);
+            for (int j = 0; j < kMaxVec; ++j) {
+                if (j >= NV) break;
+                const int at = own + 4 * P * j;
+                float g[4], gt[4], acc[4];
+                if constexpr (GDT == MTDAO_F32) {
+                    to_array(*reinterpret_cast<const float4 *>(buf + kStates * tile + at), g);
+                } else {
+                    const uint2 w =
+                        *reinterpret_cast<const uint2 *>(reinterpret_cast<const uint16_t *>(buf + kStates * tile) + at);
+                    g[0] = __uint_as_float(w.x << 16);
+                    g[1] = __uint_as_float(w.x & 0xffff0000u);
+                    g[2] = __uint_as_float(w.y << 16);
+                    g[3] = __uint_as_float(w.y & 0xffff0000u);
+                }
 #pragma unroll
-            for (int i = 0; i < kStates; ++i)
+                for (int k = 0; k < 4; ++k) acc[k] = step_acc_init<BASE>(a.sc, g[k], s);
 #pragma unroll
-                for (int j = 0; j < NV; ++j)
-                    to_array(ld_state(a.arena + state_order<BASE, N>(i) * a.stride + r * n + e + 4 * P * j),
-                             buf[i][j]);
+                for (int i = 0; i < kStates; ++i) {
+                    const int st = state_order<BASE, N>(i);
+                    float *cell = buf + slot(st) * tile + at;
+                    float cur[4];
+                    to_array(*reinterpret_cast<const float4 *>(cell), cur);
 #pragma unroll
-            for (int j = 0; j < NV; ++j)
-#pragma unroll
-                for (int k = 0; k < 4; ++k) acc[j][k] = step_acc_init<BASE>(a.sc, g[j][k], s);
-#pragma unroll
-            for (int i = 0; i < kStates; ++i) {
-                const int st = state_order<BASE, N>(i);
-                const bool due = (mask >> st) & 1u;
-                const int slot = __popc(mask & ((1u << st) - 1u));
-#pragma unroll
-                for (int j = 0; j < NV; ++j) {
-                    float *cur = buf[i][j];
-#pragma unroll
-                    for (int k = 0; k < 4; ++k)
-                        update_state<BASE, N>(a.sc, st, g[j][k], s, gt[j][k], acc[j][k], cur[k]);
-                    if (due)
-                        *reinterpret_cast<float4 *>(tile + (slot * M + r) * S + 4 * f + 4 * P * j) = from_array(cur);
+                    for (int k = 0; k < 4; ++k) update_state<BASE, N>(a.sc, st, g[k], s, gt[k], acc[k], cur[k]);
+                    if ((mask >> st) & 1u)
+                        *reinterpret_cast<float4 *>(cell) = from_array(cur);
                     else
                         st_state(a.arena + st * a.stride + r * n + e + 4 * P * j, from_array(cur));
                 }
             }
         }
         __syncthreads();
-        tile_means(tile, M, log2_p + 2 + kWideVecLog2, n_due * S, mean);
+        tile_means(buf, M, log2_s, n_due * S, mean);
         __syncthreads();
         if (live) {
 #pragma unroll
             for (int st = 0; st < kStates; ++st)
                 if ((mask >> st) & 1u) {
-                    const int slot = __popc(mask & ((1u << st) - 1u));
 #pragma unroll
-                    for (int j = 0; j < NV; ++j)
+                    for (int j = 0; j < kMaxVec; ++j) {
+                        if (j >= NV) break;
                         st_state(a.arena + st * a.stride + r * n + e + 4 * P * j,
-                                 *reinterpret_cast<const float4 *>(mean + slot * S + 4 * f + 4 * P * j));
+                                 *reinterpret_cast<const float4 *>(mean + slot(st) * S + 4 * f + 4 * P * j));
+                    }
                 }
         }
-        __syncthreads();                         // the tile and the means are reused by the next span
+        __syncthreads();                         // this buffer and the means are rewritten next
     }
+    cp_async_wait<0>();
 }
 
 template <int BASE, int N, int GDT, bool CLIP>
-cudaError_t launch_step_sync_wide(const StepArgs &a, cudaStream_t stream) {
+cudaError_t launch_step_sync_wide(const StepArgs &a, int num_sms, cudaStream_t stream) {
     if (a.M < 2 || a.M > kWideFusedMaxM) return cudaErrorNotSupported;
     const int P = wide_positions(a.M);
     int log2_p = 0;
     while ((1 << log2_p) < P) ++log2_p;
-    const int S = wide_span(a.M);
+    const int log2_v = wide_fused_vec(a.M) == 2 ? 1 : 0;
+    const int S = 4 * P << log2_v;
     const int threads = (a.M * P + 31) / 32 * 32;
     const int n_due = __builtin_popcount(a.sync_mask);
-    const size_t smem = static_cast<size_t>(n_due) * wide_floats_per_state(a.M) * sizeof(float);
+    const size_t smem = (2 * static_cast<size_t>(wide_buffer_floats<BASE, N, GDT>(a.M, S)) +
+                         static_cast<size_t>(n_due) * S) * sizeof(float);
     auto kernel = step_sync_wide_kernel<BASE, N, GDT, CLIP>;
-    if (smem > 48 * 1024) {       // above the default limit (M >= 33 with most states due)
+    if (smem > 48 * 1024) {       // above the default limit; before the occupancy query
         const cudaError_t e =
             cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
         if (e != cudaSuccess) return e;
     }
-    int64_t grid = a.n_padded / S;
-    if (grid > 0x7fffffff) grid = 0x7fffffff;
-    kernel<<<static_cast<unsigned>(grid < 1 ? 1 : grid), threads, smem, stream>>>(a, log2_p);
+    int per_sm = 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kernel, threads, smem) != cudaSuccess ||
+        per_sm < 1) {
+        cudaGetLastError();
+        per_sm = 1;
+    }
+    int64_t grid = static_cast<int64_t>(per_sm) * num_sms;
+    const int64_t n_spans = a.n_padded / S;
+    if (grid > n_spans) grid = n_spans;
+    kernel<<<static_cast<unsigned>(grid < 1 ? 1 : grid), threads, smem, stream>>>(a, log2_p, log2_v);
     return cudaGetLastError();
 }
 

@@ -137,6 +137,21 @@ WORKLOADS = {
         "init_sigma": 0.02,
         "opt": _opt("adam", (0.5, 0.9, 0.999), 0.999, 1e-3, 32, 32, 32),
     },
+    "profile_small_m16": {
+        "name": "profile_small_m16",
+        "desc": "flat fp32 vector n=2^23 with M=16 replicas and the ~1B workload's optimizer "
+                "(N=3 beta=(0.5,0.9,0.999), Adam, grads N(0,1e-3) with 1% outliers x100, "
+                "H=32): the block-staged fused step and one-pass diagnostics on ~3 GB of "
+                "device memory, for profiler captures",
+        "shapes": [1 << 23],
+        "M": 16,
+        "T": 64,
+        "grad_kind": "normal_outliers",
+        "grad_sigma": 1e-3,
+        "grad_dtype": "f32",
+        "init_sigma": 0.02,
+        "opt": _opt("adam", (0.5, 0.9, 0.999), 0.999, 1e-3, 32, 32, 32),
+    },
     "profile_small_adopt": {
         "name": "profile_small_adopt",
         "desc": "flat vector n=2^24 with the ~350M workload's optimizer (M=8, N=2 "
