@@ -61,6 +61,8 @@ def parse_args():
                     help="flat-vector sweep: one JSON line per (n, M, N) with step, fused "
                          "step+sync and sync bandwidth, and the round rate for H in {1, 8, 64}")
     ap.add_argument("--sweep-log2n", default="20,24,27,30")
+    ap.add_argument("--sweep-M", default="1,2,4,8", help="replica counts of the sweep")
+    ap.add_argument("--sweep-N", default="1,2,3,4", help="momentum counts of the sweep")
     ap.add_argument("--second-workload", default="decoder_350m",
                     help="workload timed in a child process after the main one ('' = none)")
     return ap.parse_args()
@@ -602,8 +604,8 @@ def run_child_workload(name: str, steps: int, warmup: int):
 
 
 def run_sweep(args):
-    """Flat fp32 vector n = 2^k, M in {1,2,4,8}, N in {1..4} (Adam, f32
-    gradients).  Each (n, M, N) point times 6 launches (2 warm-up) of the
+    """Flat fp32 vector n = 2^k, M in --sweep-M (default {1,2,4,8}), N in
+    --sweep-N (default {1..4}) (Adam, f32 gradients).  Each (n, M, N) point times 6 launches (2 warm-up) of the
     plain step, the fused step + average of every state, and the standalone
     average; per H in {1, 8, 64} a round is (H-1) plain steps and one fused
     step, so its rate follows from those times."""
@@ -635,8 +637,8 @@ def run_sweep(args):
         return statistics.median(out)
 
     for k in [int(v) for v in args.sweep_log2n.split(",")]:
-        for M in (1, 2, 4, 8):
-            for N in (1, 2, 3, 4):
+        for M in [int(v) for v in args.sweep_M.split(",")]:
+            for N in [int(v) for v in args.sweep_N.split(",")]:
                 w = W.sweep_point(k, M, N, 8)
                 n_states = N + 2
                 need = M * (1 << k) * (4 * n_states + 4) + (4 << 30)

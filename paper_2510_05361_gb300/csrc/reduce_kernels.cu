@@ -25,13 +25,49 @@ namespace mtdao {
 
 namespace {
 
+// Mean of the M replicas at float4 position e of state s, M known at run
+// time (the standalone average above 8 replicas and the two-pass
+// diagnostics): replica_mean.cuh's operations in its order, four replicas'
+// loads in flight (one at a time, the average of M = 9-64 ran at 5.5-5.8
+// TB/s).
+__device__ __forceinline__ float4 replica_mean4(const float *s, int64_t n, int M, int64_t e) {
+    float s0[4];
+    to_array(ld_state(s + e), s0);
+    DiffSum pa[4] = {DiffSum(s0[0]), DiffSum(s0[1]), DiffSum(s0[2]), DiffSum(s0[3])};
+    DiffSum pb[4] = {DiffSum(s0[0]), DiffSum(s0[1]), DiffSum(s0[2]), DiffSum(s0[3])};
+    float plain[4] = {s0[0], s0[1], s0[2], s0[3]};
+    const int h = M / 2;
+    for (int m = 1; m < M; m += 4) {          // four replicas' loads in flight, added in order
+        float r[4][4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u)
+            if (m + u < M) to_array(ld_state(s + (m + u) * n + e), r[u]);
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            if (m + u >= M) break;
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+                if (m + u < h) pa[k].add(r[u][k]);
+                else pb[k].add(r[u][k]);
+                plain[k] += r[u][k];
+            }
+        }
+    }
+    float mean[4];
+#pragma unroll
+    for (int k = 0; k < 4; ++k)
+        mean[k] = mean_or_plain(
+            replica_mean_from_parts(s0[k], pa[k].partial(), pb[k].partial(), static_cast<float>(M)), plain[k],
+            static_cast<float>(M));
+    return from_array(mean);
+}
+
 template <int MT>
 __global__ void __launch_bounds__(kThreads) sync_kernel(const SyncArgs a) {
     const int M = MT > 0 ? MT : a.M;
     float *base = a.arena + static_cast<int64_t>(a.sel[blockIdx.y]) * a.stride;
     const int64_t n = a.n_padded;
     const int64_t nv = n / 4;
-    const float Mf = static_cast<float>(M);
     for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < nv;
          i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
         const int64_t e = 4 * i;
@@ -44,26 +80,7 @@ __global__ void __launch_bounds__(kThreads) sync_kernel(const SyncArgs a) {
             for (int k = 0; k < 4; ++k) mean[k] = replica_mean<MT>([&](int m) { return r[m][k]; });
         } else {
             // streamed: replicas 1 .. h-1 feed part A, h .. M-1 part B (replica_mean.cuh)
-            float s0[4];
-            to_array(ld_state(base + e), s0);
-            DiffSum pa[4] = {DiffSum(s0[0]), DiffSum(s0[1]), DiffSum(s0[2]), DiffSum(s0[3])};
-            DiffSum pb[4] = {DiffSum(s0[0]), DiffSum(s0[1]), DiffSum(s0[2]), DiffSum(s0[3])};
-            float plain[4] = {s0[0], s0[1], s0[2], s0[3]};
-            const int h = M / 2;
-            for (int m = 1; m < M; ++m) {
-                float r[4];
-                to_array(ld_state(base + m * n + e), r);
-#pragma unroll
-                for (int k = 0; k < 4; ++k) {
-                    if (m < h) pa[k].add(r[k]);
-                    else pb[k].add(r[k]);
-                    plain[k] += r[k];
-                }
-            }
-#pragma unroll
-            for (int k = 0; k < 4; ++k)
-                mean[k] = mean_or_plain(replica_mean_from_parts(s0[k], pa[k].partial(), pb[k].partial(), Mf),
-                                        plain[k], Mf);
+            to_array(replica_mean4(base, n, M, e), mean);
         }
         const float4 mv = from_array(mean);
         for (int m = 0; m < M; ++m) st_state(base + m * n + e, mv);
@@ -72,11 +89,14 @@ __global__ void __launch_bounds__(kThreads) sync_kernel(const SyncArgs a) {
 
 template <int MT>
 cudaError_t launch_sync_t(const SyncArgs &a, int num_sms, cudaStream_t stream) {
-    // M = 2, 4, 8 (replicas held in registers): one float4 position per
+    // M = 2 .. 14 (replicas held in registers): one float4 position per
     // thread, like the local step's stream_grid (flat 2^27, all states, GB/s
     // against the persistent grid: M = 2 6342 -> 7098, M = 4 6447 -> 7025,
-    // M = 8 6546 -> 6941).  The streamed runtime-M loop keeps the persistent
-    // grid (M = 3: 6257, one position per thread 5591).
+    // M = 8 6546 -> 6941; flat 2^30 replica-elements against the streamed
+    // loop: M = 3 4588 -> 6336, 5-7 5069 -> 6609-6658, 9-14 5564 -> 6343-6784).
+    // At 15 and 16 the replicas take 151-176 registers (M = 16: 5086 against
+    // 5796 streamed).  The streamed runtime-M loop (M > 14) keeps the
+    // persistent grid (one position per thread: 3-7 % slower at M = 9-64).
     const int64_t nv = a.n_padded / 4;
     const int64_t need = (nv + kThreads - 1) / kThreads;
     int64_t gx;
@@ -490,40 +510,6 @@ __device__ void block_sum_k(const double (&v)[K], double *out) {
     }
 }
 
-// Mean of the M replicas at float4 position e of state s: the runtime-M
-// form of sync_kernel, the same operations in the same order.
-__device__ __forceinline__ float4 replica_mean4(const float *s, int64_t n, int M, int64_t e) {
-    float s0[4];
-    to_array(ld_state(s + e), s0);
-    DiffSum pa[4] = {DiffSum(s0[0]), DiffSum(s0[1]), DiffSum(s0[2]), DiffSum(s0[3])};
-    DiffSum pb[4] = {DiffSum(s0[0]), DiffSum(s0[1]), DiffSum(s0[2]), DiffSum(s0[3])};
-    float plain[4] = {s0[0], s0[1], s0[2], s0[3]};
-    const int h = M / 2;
-    for (int m = 1; m < M; m += 4) {          // four replicas' loads in flight, added in order
-        float r[4][4];
-#pragma unroll
-        for (int u = 0; u < 4; ++u)
-            if (m + u < M) to_array(ld_state(s + (m + u) * n + e), r[u]);
-#pragma unroll
-        for (int u = 0; u < 4; ++u) {
-            if (m + u >= M) break;
-#pragma unroll
-            for (int k = 0; k < 4; ++k) {
-                if (m + u < h) pa[k].add(r[u][k]);
-                else pb[k].add(r[u][k]);
-                plain[k] += r[u][k];
-            }
-        }
-    }
-    float mean[4];
-#pragma unroll
-    for (int k = 0; k < 4; ++k)
-        mean[k] = mean_or_plain(
-            replica_mean_from_parts(s0[k], pa[k].partial(), pb[k].partial(), static_cast<float>(M)), plain[k],
-            static_cast<float>(M));
-    return from_array(mean);
-}
-
 // Positions a pass-2 thread loads before it accumulates them (i, i + T,
 // i + 2T, ...: the order of a plain grid-stride loop): four for the sync
 // diagnostics (two float4 loads per position), two for the change
@@ -756,8 +742,18 @@ cudaError_t launch_sync(const SyncArgs &a, int num_sms, cudaStream_t stream) {
     if (a.n_sel <= 0 || a.M <= 1) return cudaSuccess;
     switch (a.M) {
         case 2: return launch_sync_t<2>(a, num_sms, stream);
+        case 3: return launch_sync_t<3>(a, num_sms, stream);
         case 4: return launch_sync_t<4>(a, num_sms, stream);
+        case 5: return launch_sync_t<5>(a, num_sms, stream);
+        case 6: return launch_sync_t<6>(a, num_sms, stream);
+        case 7: return launch_sync_t<7>(a, num_sms, stream);
         case 8: return launch_sync_t<8>(a, num_sms, stream);
+        case 9: return launch_sync_t<9>(a, num_sms, stream);
+        case 10: return launch_sync_t<10>(a, num_sms, stream);
+        case 11: return launch_sync_t<11>(a, num_sms, stream);
+        case 12: return launch_sync_t<12>(a, num_sms, stream);
+        case 13: return launch_sync_t<13>(a, num_sms, stream);
+        case 14: return launch_sync_t<14>(a, num_sms, stream);
         default: return launch_sync_t<0>(a, num_sms, stream);
     }
 }

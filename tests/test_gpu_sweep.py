@@ -1,5 +1,6 @@
 """Parity on points of the flat-vector sweep workload (n = 2^20, M in
-{1,2,4,8}, N in {1..4}, H in {1,8,64}, including the base-optimizer
+{1,2,4,8} and four points with 12 to 64 replicas, N in {1..4}, H in
+{1,8,64}, including the base-optimizer
 reduction point N=1, omega=1, H=1): T = 3H local steps (8 for H = 1) with
 device-generated gradients, the oracle on a sample of elements."""
 import numpy as np
@@ -14,7 +15,8 @@ pytestmark = pytest.mark.gpu
 
 POINTS = ([(M, N, 8) for M in (1, 2, 4, 8) for N in (1, 2, 3, 4)]
           + [(M, 1, 1) for M in (1, 2, 4, 8)]
-          + [(4, 2, 64), (8, 4, 64), (2, 3, 1)])
+          + [(4, 2, 64), (8, 4, 64), (2, 3, 1)]
+          + [(12, 1, 8), (16, 3, 8), (32, 2, 8), (64, 4, 1)])   # the block-staged fused step
 
 
 @pytest.fixture(scope="module")
