@@ -60,6 +60,7 @@ __device__ __forceinline__ void fetch_row(bool live, float *dst, const float *sr
 //   q = 2 + M + m  sum_i s_m * s_bar
 // at partial[(blockIdx.y * gridDim.x + blockIdx.x) * Q + q], Q = 2 + 2M;
 // s_bar (the fp32 mean) is written over every replica.
+template <bool FOUR>
 __global__ void __launch_bounds__(kWideMaxThreads) sync_stats_wide_kernel(const SyncArgs a, int log2_p,
                                                                           double *partial) {
     extern __shared__ __align__(16) float smem[];
@@ -90,7 +91,7 @@ __global__ void __launch_bounds__(kWideMaxThreads) sync_stats_wide_kernel(const 
         cp_async_wait<1>();                      // this thread's copies of `span` have landed
         __syncthreads();                         // ... and every thread's
         const float *tile = tiles + buf * M * S;
-        tile_means(tile, M, log2_s, S, mean);
+        tile_means<FOUR>(tile, M, log2_s, S, mean);
         __syncthreads();
         if (live) {
             float p0 = 0.0f, p1 = 0.0f, p2 = 0.0f, p3 = 0.0f;   // this thread's 4 * NV elements
@@ -157,6 +158,7 @@ __global__ void __launch_bounds__(kWideMaxThreads) sync_stats_wide_kernel(const 
 //   q = 2M         sum_i (x_bar - a)^2
 //   q = 2M + 1     sum_i a^2
 // The anchor's span travels with replica 0's row (one more tile row).
+template <bool FOUR>
 __global__ void __launch_bounds__(kWideMaxThreads) pseudo_grad_stats_wide_kernel(const float *x,
                                                                                  const float *anchor,
                                                                                  int64_t n, int M, int log2_p,
@@ -194,7 +196,7 @@ __global__ void __launch_bounds__(kWideMaxThreads) pseudo_grad_stats_wide_kernel
         __syncthreads();
         const float *tile = tiles + buf * R * S;
         const float *anc = tile + M * S;
-        tile_means(tile, M, log2_s, S, mean);
+        tile_means<FOUR>(tile, M, log2_s, S, mean);
         __syncthreads();
         if (live) {
             float p0 = 0.0f, p1 = 0.0f, p2 = 0.0f, p3 = 0.0f;   // this thread's 4 * NV elements
@@ -304,46 +306,66 @@ size_t wide_stats_partial_capacity(int num_sms, int n_states, int M) {
     return static_cast<size_t>(32 * num_sms + n_states) * (2 + 2 * static_cast<size_t>(M));
 }
 
-cudaError_t launch_sync_stats_wide(const SyncArgs &a, int num_sms, double *partial, size_t partial_cap,
-                                   double *stats, cudaStream_t stream) {
+namespace {
+
+template <bool FOUR>
+cudaError_t launch_sync_stats_wide_t(const SyncArgs &a, int num_sms, double *partial, size_t partial_cap,
+                                     double *stats, cudaStream_t stream) {
     if (a.n_sel <= 0) return cudaSuccess;
     if (a.M < 2 || a.M > kWideMaxM) return cudaErrorNotSupported;
     const int Q = 2 + 2 * a.M;
     const WideShape w = wide_shape(a.M, 0);
     if (w.smem > 48 * 1024) {        // before the occupancy query, which depends on it
-        cudaError_t e = cudaFuncSetAttribute(sync_stats_wide_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+        cudaError_t e = cudaFuncSetAttribute(sync_stats_wide_kernel<FOUR>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                              static_cast<int>(w.smem));
         if (e != cudaSuccess) return e;
     }
-    const int per_sm = wide_blocks_per_sm(sync_stats_wide_kernel, w);
+    const int per_sm = wide_blocks_per_sm(sync_stats_wide_kernel<FOUR>, w);
     if (static_cast<size_t>(Q) * a.n_sel > partial_cap) return cudaErrorInvalidValue;
     const int g = wide_grid(per_sm, num_sms, a.n_sel, a.n_padded / w.S, Q, partial_cap);
-    sync_stats_wide_kernel<<<dim3(g, a.n_sel), w.threads, w.smem, stream>>>(a, w.log2_p, partial);
+    sync_stats_wide_kernel<FOUR><<<dim3(g, a.n_sel), w.threads, w.smem, stream>>>(a, w.log2_p, partial);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
     wide_stats_finalize_kernel<<<dim3((Q + 255) / 256, a.n_sel), 256, 0, stream>>>(partial, g, Q, a.M, stats);
     return cudaGetLastError();
 }
 
-cudaError_t launch_pseudo_grad_stats_wide(const float *x, const float *anchor, int64_t n, int M, int num_sms,
-                                          double *partial, size_t partial_cap, double *stats,
-                                          cudaStream_t stream) {
+template <bool FOUR>
+cudaError_t launch_pseudo_grad_stats_wide_t(const float *x, const float *anchor, int64_t n, int M, int num_sms,
+                                            double *partial, size_t partial_cap, double *stats,
+                                            cudaStream_t stream) {
     if (M < 2 || M > kWideMaxM) return cudaErrorNotSupported;
     const int Q = 2 * M + 2;
     const WideShape w = wide_shape(M, 1);
     if (w.smem > 48 * 1024) {        // before the occupancy query, which depends on it
-        cudaError_t e = cudaFuncSetAttribute(pseudo_grad_stats_wide_kernel,
+        cudaError_t e = cudaFuncSetAttribute(pseudo_grad_stats_wide_kernel<FOUR>,
                                              cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(w.smem));
         if (e != cudaSuccess) return e;
     }
-    const int per_sm = wide_blocks_per_sm(pseudo_grad_stats_wide_kernel, w);
+    const int per_sm = wide_blocks_per_sm(pseudo_grad_stats_wide_kernel<FOUR>, w);
     if (static_cast<size_t>(Q) > partial_cap) return cudaErrorInvalidValue;
     const int g = wide_grid(per_sm, num_sms, 1, n / w.S, Q, partial_cap);
-    pseudo_grad_stats_wide_kernel<<<g, w.threads, w.smem, stream>>>(x, anchor, n, M, w.log2_p, partial);
+    pseudo_grad_stats_wide_kernel<FOUR><<<g, w.threads, w.smem, stream>>>(x, anchor, n, M, w.log2_p, partial);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
     wide_stats_finalize_kernel<<<dim3((Q + 255) / 256, 1), 256, 0, stream>>>(partial, g, Q, 0, stats);
     return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t launch_sync_stats_wide(const SyncArgs &a, int num_sms, double *partial, size_t partial_cap,
+                                   double *stats, cudaStream_t stream) {
+    return wide_four_columns(a.M) ? launch_sync_stats_wide_t<true>(a, num_sms, partial, partial_cap, stats, stream)
+                                  : launch_sync_stats_wide_t<false>(a, num_sms, partial, partial_cap, stats, stream);
+}
+
+cudaError_t launch_pseudo_grad_stats_wide(const float *x, const float *anchor, int64_t n, int M, int num_sms,
+                                          double *partial, size_t partial_cap, double *stats,
+                                          cudaStream_t stream) {
+    return wide_four_columns(M)
+               ? launch_pseudo_grad_stats_wide_t<true>(x, anchor, n, M, num_sms, partial, partial_cap, stats, stream)
+               : launch_pseudo_grad_stats_wide_t<false>(x, anchor, n, M, num_sms, partial, partial_cap, stats, stream);
 }
 
 }  // namespace mtdao

@@ -41,14 +41,63 @@ constexpr int wide_positions(int M) { return M <= 16 ? 16 : M <= 64 ? 8 : M <= 1
 
 // Replica means of the n_cols columns of a block's tile into mean[p]
 // (column p: tile + (p / S) * M * S + p % S, the replicas at stride
-// S = 2^log2_s; shifts, not a division by a run-time S).
-// Lanes 2i and 2i + 1 form the two compensated parts of replica_mean.cuh
-// for one column, replicas 1 .. h-1 and h .. M-1 in order (h = M / 2), and
-// join them with a shuffle: the bits of replica_mean_rt (with its plain
-// mean where the compensated one is NaN).  Every thread of
-// the block calls it (the shuffles take whole warps: blockDim.x is a
-// multiple of 32 and the loop count is the same for all threads).
-__device__ __forceinline__ void tile_means(const float *tile, int M, int log2_s, int n_cols, float *mean) {
+// S = 2^log2_s; shifts, not a division by a run-time S).  Columns go in
+// groups of four (n_cols and S are multiples of 4): lanes 2i and 2i + 1
+// take one group and form its two compensated parts of replica_mean.cuh,
+// replicas 1 .. h-1 and h .. M-1 in order (h = M / 2), four columns at a
+// time from one 16-byte shared load per replica, and join them with
+// shuffles: the bits of replica_mean_rt (with its plain mean where the
+// compensated one is NaN).  Every thread of the block calls it (the
+// shuffles take whole warps: blockDim.x is a multiple of 32 and the loop
+// count is the same for all threads).
+__device__ __forceinline__ void tile_means4(const float *tile, int M, int log2_s, int n_cols, float *mean) {
+    const int t = threadIdx.x;
+    const int h = M / 2;
+    const int S = 1 << log2_s;
+    const int n_tasks = n_cols / 2;              // (group of four columns, part) pairs
+    for (int q0 = 0; q0 < n_tasks; q0 += static_cast<int>(blockDim.x)) {
+        const int q = q0 + t;
+        const int part = q & 1;
+        const int p = 4 * (q >> 1);              // first column of the group
+        const float *base = tile + (p >> log2_s) * M * S + (p & (S - 1));
+        float s0[4] = {0.0f, 0.0f, 0.0f, 0.0f}, mine[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+        if (q < n_tasks) {
+            to_array(*reinterpret_cast<const float4 *>(base), s0);
+            DiffSum sum[4] = {DiffSum(s0[0]), DiffSum(s0[1]), DiffSum(s0[2]), DiffSum(s0[3])};
+            const int lo = part ? h : 1, hi = part ? M : h;
+#pragma unroll 2
+            for (int m = lo; m < hi; ++m) {
+                float v[4];
+                to_array(*reinterpret_cast<const float4 *>(base + m * S), v);
+#pragma unroll
+                for (int k = 0; k < 4; ++k) sum[k].add(v[k]);
+            }
+#pragma unroll
+            for (int k = 0; k < 4; ++k) mine[k] = sum[k].partial();
+        }
+        float other[4];
+#pragma unroll
+        for (int k = 0; k < 4; ++k) other[k] = __shfl_xor_sync(0xffffffffu, mine[k], 1);
+        if (q < n_tasks && part == 0) {
+            float v[4];
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+                v[k] = replica_mean_from_parts(s0[k], mine[k], other[k], static_cast<float>(M));
+                if (v[k] != v[k]) {              // non-finite values: the plain mean (replica_mean.cuh)
+                    float plain = s0[k];
+                    for (int m = 1; m < M; ++m) plain += base[m * S + k];
+                    v[k] = plain / static_cast<float>(M);
+                }
+            }
+            *reinterpret_cast<float4 *>(mean + p) = from_array(v);
+        }
+    }
+}
+
+// The same means one column per lane pair (lanes 2i and 2i + 1 run the two
+// parts of column i with 4-byte shared loads): more lanes at work on fewer
+// columns each, which is the better trade for M above 32.
+__device__ __forceinline__ void tile_means1(const float *tile, int M, int log2_s, int n_cols, float *mean) {
     const int t = threadIdx.x;
     const int h = M / 2;
     const int S = 1 << log2_s;
@@ -56,8 +105,8 @@ __device__ __forceinline__ void tile_means(const float *tile, int M, int log2_s,
         const int p = p0 + (t >> 1);
         const int part = t & 1;
         float s0 = 0.0f, mine = 0.0f;
+        const float *col = tile + (p >> log2_s) * M * S + (p & (S - 1));
         if (p < n_cols) {
-            const float *col = tile + (p >> log2_s) * M * S + (p & (S - 1));
             s0 = col[0];
             DiffSum sum(s0);
             const int lo = part ? h : 1, hi = part ? M : h;
@@ -69,14 +118,29 @@ __device__ __forceinline__ void tile_means(const float *tile, int M, int log2_s,
         if (p < n_cols && part == 0) {
             float v = replica_mean_from_parts(s0, mine, other, static_cast<float>(M));
             if (v != v) {                        // non-finite values: the plain mean (replica_mean.cuh)
-                const float *col = tile + (p >> log2_s) * M * S + (p & (S - 1));
-                float plain = col[0];
+                float plain = s0;
                 for (int m = 1; m < M; ++m) plain += col[m * S];
                 v = plain / static_cast<float>(M);
             }
             mean[p] = v;
         }
     }
+}
+
+// The per-span means of the wide kernels: four columns per lane pair up to
+// M = 32 (flat sweep, fused step, N = 3: M = 9 4861 -> 5825 GB/s, 24-32
+// 5397-5458 -> 5908-5915), one above (M = 64: 4998 against 4887 with four,
+// where only n_cols / 2 of up to 512 threads have work).  A compile-time
+// choice: with both forms in one kernel the fused step took 101-108
+// registers instead of 50-64 and lost occupancy.
+constexpr bool wide_four_columns(int M) { return M <= 32; }
+
+template <bool FOUR>
+__device__ __forceinline__ void tile_means(const float *tile, int M, int log2_s, int n_cols, float *mean) {
+    if constexpr (FOUR)
+        tile_means4(tile, M, log2_s, n_cols, mean);
+    else
+        tile_means1(tile, M, log2_s, n_cols, mean);
 }
 
 // 16- and 8-byte asynchronous global -> shared copies (cp.async) and their
@@ -115,7 +179,7 @@ __host__ __device__ constexpr int wide_buffer_floats(int M, int S) {
 // one block fitted per SM: M = 48 and 64 fell from 4.9-5.0 to 3.9-4.2 TB/s.
 constexpr int wide_fused_vec(int M) { return (M > 16 && M <= 32) ? 2 : 1; }
 
-template <int BASE, int N, int GDT, bool CLIP>
+template <int BASE, int N, int GDT, bool CLIP, bool FOUR>
 __global__ void __launch_bounds__(kWideMaxThreads) step_sync_wide_kernel(const StepArgs a, int log2_p,
                                                                          int log2_v) {
     extern __shared__ __align__(16) float smem[];
@@ -209,7 +273,7 @@ __global__ void __launch_bounds__(kWideMaxThreads) step_sync_wide_kernel(const S
             }
         }
         __syncthreads();
-        tile_means(buf, M, log2_s, n_due * S, mean);
+        tile_means<FOUR>(buf, M, log2_s, n_due * S, mean);
         __syncthreads();
         if (live) {
 #pragma unroll
@@ -228,8 +292,8 @@ __global__ void __launch_bounds__(kWideMaxThreads) step_sync_wide_kernel(const S
     cp_async_wait<0>();
 }
 
-template <int BASE, int N, int GDT, bool CLIP>
-cudaError_t launch_step_sync_wide(const StepArgs &a, int num_sms, cudaStream_t stream) {
+template <int BASE, int N, int GDT, bool CLIP, bool FOUR>
+cudaError_t launch_step_sync_wide_t(const StepArgs &a, int num_sms, cudaStream_t stream) {
     if (a.M < 2 || a.M > kWideFusedMaxM) return cudaErrorNotSupported;
     const int P = wide_positions(a.M);
     int log2_p = 0;
@@ -240,7 +304,7 @@ cudaError_t launch_step_sync_wide(const StepArgs &a, int num_sms, cudaStream_t s
     const int n_due = __builtin_popcount(a.sync_mask);
     const size_t smem = (2 * static_cast<size_t>(wide_buffer_floats<BASE, N, GDT>(a.M, S)) +
                          static_cast<size_t>(n_due) * S) * sizeof(float);
-    auto kernel = step_sync_wide_kernel<BASE, N, GDT, CLIP>;
+    auto kernel = step_sync_wide_kernel<BASE, N, GDT, CLIP, FOUR>;
     if (smem > 48 * 1024) {       // above the default limit; before the occupancy query
         const cudaError_t e =
             cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
@@ -257,6 +321,12 @@ cudaError_t launch_step_sync_wide(const StepArgs &a, int num_sms, cudaStream_t s
     if (grid > n_spans) grid = n_spans;
     kernel<<<static_cast<unsigned>(grid < 1 ? 1 : grid), threads, smem, stream>>>(a, log2_p, log2_v);
     return cudaGetLastError();
+}
+
+template <int BASE, int N, int GDT, bool CLIP>
+cudaError_t launch_step_sync_wide(const StepArgs &a, int num_sms, cudaStream_t stream) {
+    return wide_four_columns(a.M) ? launch_step_sync_wide_t<BASE, N, GDT, CLIP, true>(a, num_sms, stream)
+                                  : launch_step_sync_wide_t<BASE, N, GDT, CLIP, false>(a, num_sms, stream);
 }
 
 }  // namespace mtdao
