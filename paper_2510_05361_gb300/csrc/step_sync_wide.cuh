@@ -18,12 +18,13 @@
 // loop), in the same order, so fused and separate averaging give identical
 // bits for every M.
 //
-// Rows of the span are 32 bytes or longer: P = 16 (M <= 16), 8 (M <= 64),
-// 4 (M <= 128), 2 (M <= 256) float4 positions per thread row, so a block
-// has M * P <= 512 threads (rounded up to whole warps; threads beyond M * P
-// only take part in the mean).  Shared memory of the fused step: two span
-// buffers (a tile per state and the gradient tile) and S means per due
-// state.
+// A replica's row of a span is handled by P threads: P = 16 (M <= 16), 8
+// (M <= 64), 4 (M <= 128), 2 (M <= 256), so a block has M * P <= 512
+// threads (rounded up to whole warps; threads beyond M * P only take part
+// in the mean).  The fused step's rows are 64 elements (256 bytes) up to
+// M = 32 and 32 above; the one-pass diagnostics' rows are 16 P elements.
+// Shared memory of the fused step: two span buffers (a tile per state and
+// the gradient tile) and S means per due state.
 #pragma once
 
 #include "replica_mean.cuh"
@@ -164,13 +165,6 @@ __host__ __device__ constexpr int wide_buffer_floats(int M, int S) {
     return kNumStates<BASE, N> * M * S + (GDT == MTDAO_F32 ? M * S : M * S / 2);
 }
 
-// The fused step on spans of all replicas, persistent, double-buffered:
-// while a block updates span i from shared memory, span i + gridDim.x of
-// every state and of the gradient is on its way in (cp.async).  In a
-// buffer the due states' tiles come first (in state index order), so the
-// means read them as one [n_due][M][S] array; a due state's updated values
-// are written back over its own tile, a state that is not due goes
-// straight to HBM.
 // Float4 positions per thread and row of the fused step's span (the
 // positions f and f + P): rows of 256 bytes up to M = 32 (S = 64).  With one
 // position and P = 8 (rows of 128 bytes) M = 24 and 32 ran at 4.8-4.9 TB/s
@@ -179,6 +173,13 @@ __host__ __device__ constexpr int wide_buffer_floats(int M, int S) {
 // one block fitted per SM: M = 48 and 64 fell from 4.9-5.0 to 3.9-4.2 TB/s.
 constexpr int wide_fused_vec(int M) { return (M > 16 && M <= 32) ? 2 : 1; }
 
+// The fused step on spans of all replicas, persistent, double-buffered:
+// while a block updates span i from shared memory, span i + gridDim.x of
+// every state and of the gradient is on its way in (cp.async).  In a
+// buffer the due states' tiles come first (in state index order), so the
+// means read them as one [n_due][M][S] array; a due state's updated values
+// are written back over its own tile, a state that is not due goes
+// straight to HBM.
 template <int BASE, int N, int GDT, bool CLIP, bool FOUR>
 __global__ void __launch_bounds__(kWideMaxThreads) step_sync_wide_kernel(const StepArgs a, int log2_p,
                                                                          int log2_v) {
