@@ -1,10 +1,12 @@
 // stats_wide.cu -- the cross-worker diagnostics of section 4.1 in one pass
-// for 9 <= M <= kWideMaxM replicas (the register-resident kernels of
-// reduce_kernels.cu hold up to 8).
+// for 9 <= M <= 64 replicas (the kernels take up to kWideMaxM = 256; above
+// 64 the library uses the two-pass form of reduce_kernels.cu, whose
+// register-resident kernels cover M <= 8).
 //
 // Same block layout as the wide fused step (step_sync_wide.cuh): a block
 // owns spans of S consecutive elements of all M replicas, thread (r, f)
-// loads elements [4f, 4f + 4) of replica r into a shared M x S tile, the
+// copies 16 elements of replica r (four float4 positions f, f + P, ...) into
+// a shared M x S tile (double-buffered with cp.async), the
 // span's replica means are formed from the tile by tile_means (the bits of
 // the standalone average), and each thread then forms its own replica's
 // sums against the mean.  Every replica value is read from HBM once; the
