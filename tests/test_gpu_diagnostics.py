@@ -33,11 +33,11 @@ def _fill(eng, rng, spread):
     return vals
 
 
-@pytest.mark.parametrize("M", [1, 2, 3, 4, 8, 9, 16, 37, 100, 256, 300])
+@pytest.mark.parametrize("M", [1, 2, 3, 4, 8, 9, 16, 32, 33, 37, 64, 65, 100, 256, 300])
 def test_sync_stats_match_oracle_and_plain_sync(P, M):
-    """M <= 8: one pass with the replicas in registers; 9 <= M <= 256: one
-    pass with a span of all replicas staged in shared memory; M > 256: two
-    passes through a scratch mean.  All match the oracle's definitions and
+    """M <= 8: one pass with the replicas in registers; 9 <= M <= 64: one
+    pass with a span of all replicas staged in shared memory (four-column
+    means up to 32); M > 64: two passes through a scratch mean.  All match the oracle's definitions and
     leave the states bit-identical to the plain average."""
     shapes = [70001, 999, 4096] if M <= 37 else [7001, 99, 1024]
     w = workload_dict(shapes, M, betas=(0.9, 0.99))
@@ -105,7 +105,7 @@ def test_sync_stats_rejects_bad_masks(P):
     eng.close()
 
 
-@pytest.mark.parametrize("M", [2, 4, 8, 9, 16, 37, 256, 300])
+@pytest.mark.parametrize("M", [2, 4, 8, 9, 16, 32, 33, 37, 64, 65, 256, 300])
 def test_pseudo_grad_stats_against_oracle(P, M):
     """Anchor = parameters at the last average; mid-round diagnostics of the
     pseudo-gradients match the oracle's definitions on the same values."""

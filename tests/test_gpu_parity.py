@@ -110,6 +110,27 @@ def test_fused_sync_is_bitwise_equal_to_separate_sync(P, M, gdt):
         b.close()
 
 
+@pytest.mark.parametrize("M", range(2, 71))
+def test_fused_equals_separate_for_every_replica_count(P, M):
+    """Every M from 2 to 70 crosses each switch between averaging paths:
+    lane groups (M <= 8), the block-staged fused step (9..64; one or two
+    float4 positions per thread at 16/17, four-column or one-column means at
+    32/33), step + average above 64, and the standalone average in registers
+    (M <= 14) or streamed.  Fused and separate averaging agree bit for bit,
+    and the averaged states equal the oracle within the tolerance."""
+    w = workload_dict([700, 300, 24], M, base="adam", betas=(0.9, 0.99), px=2, pu=[3, 2], pv=3, gdt="f32")
+    a = gpu_run(P, w, 6, fused=True)
+    b = gpu_run(P, w, 6, fused=False)
+    sa, sb = gpu_states(a, w["opt"]), gpu_states(b, w["opt"])
+    for k in sa:
+        assert np.array_equal(sa[k].view(np.uint32), sb[k].view(np.uint32)), k
+    lay = W.layout(w["shapes"])
+    ref = oracle_run(w["opt"], M, np.arange(lay["n_padded"]), 6, lay, w, SEED_G, SEED_I)
+    compare(sa, ref)
+    a.close()
+    b.close()
+
+
 @pytest.mark.parametrize("M", [3, 4, 5, 7, 8, 12, 16, 32])
 @pytest.mark.parametrize("gdt", ["f32", "bf16"])
 @pytest.mark.parametrize("base", ["adam", "sgdm"])
