@@ -28,7 +28,7 @@ def P():
     return P
 
 
-def draw(case):
+def draw(case, replica_counts=None):
     rng = np.random.default_rng(1000 + case)
     base = ["adam", "adopt", "sgdm"][case % 3]
     N = int(rng.integers(1, 5))
@@ -45,6 +45,8 @@ def draw(case):
     if base != "adopt" and rng.random() < 0.3:
         clip = "global_norm"
     M = int(rng.choice([1, 2, 3, 4, 5, 6, 7, 8, 9, 12, 16, 32]))
+    if replica_counts is not None:
+        M = int(rng.choice(replica_counts))
     shapes = [int(rng.choice([0, 1, 7, 64, 333, 1000, 4099])) for _ in range(int(rng.integers(1, 6)))]
     if sum(shapes) == 0:
         shapes.append(513)
@@ -63,9 +65,7 @@ def draw(case):
     return w, int(rng.integers(3, 17))
 
 
-@pytest.mark.parametrize("case", range(96))
-def test_random_configuration_parity(P, case):
-    w, T = draw(case)
+def run_case(P, w, T):
     opt, M = w["opt"], w["M"]
     lay = W.layout(w["shapes"])
     n = lay["n_padded"]
@@ -80,3 +80,15 @@ def test_random_configuration_parity(P, case):
     got = {nm: eng.state_view(s).cpu().numpy() for s, nm in enumerate(names)}
     eng.close()
     compare(got, oracle_run(opt, M, idx, T, lay, w, SEED_G, SEED_I))
+
+
+@pytest.mark.parametrize("case", range(96))
+def test_random_configuration_parity(P, case):
+    run_case(P, *draw(case))
+
+
+@pytest.mark.parametrize("case", range(96, 120))
+def test_random_configuration_parity_wide(P, case):
+    """The same draws with replica counts on both sides of the block-staged
+    fused step's layout switches (10, 24, 40, 64)."""
+    run_case(P, *draw(case, replica_counts=[10, 24, 40, 64]))
