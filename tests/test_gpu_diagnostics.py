@@ -33,7 +33,7 @@ def _fill(eng, rng, spread):
     return vals
 
 
-@pytest.mark.parametrize("M", [1, 2, 3, 4, 8, 9, 16, 32, 33, 37, 64, 65, 100, 256, 300])
+@pytest.mark.parametrize("M", [1, 2, 3, 4, 8, 9, 16, 32, 33, 37, 64, 65, 100, 256, 300, 1024])
 def test_sync_stats_match_oracle_and_plain_sync(P, M):
     """M <= 8: one pass with the replicas in registers; 9 <= M <= 64: one
     pass with a span of all replicas staged in shared memory (four-column
@@ -105,7 +105,7 @@ def test_sync_stats_rejects_bad_masks(P):
     eng.close()
 
 
-@pytest.mark.parametrize("M", [2, 4, 8, 9, 16, 32, 33, 37, 64, 65, 256, 300])
+@pytest.mark.parametrize("M", [2, 4, 8, 9, 16, 32, 33, 37, 64, 65, 256, 300, 1024])
 def test_pseudo_grad_stats_against_oracle(P, M):
     """Anchor = parameters at the last average; mid-round diagnostics of the
     pseudo-gradients match the oracle's definitions on the same values."""
