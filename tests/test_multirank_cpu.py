@@ -137,3 +137,19 @@ def test_clock_sample_summary():
     assert s["reasons"] == ["hw_slowdown", "sw_power_cap"]
     assert s["sm_mhz"] == statistics.median([2070.0, 1890.0, 1890.0, 1500.0])
     assert bench.parse_clock_samples([])["reasons"] == ["no samples"]
+
+
+def test_sweep_options(monkeypatch):
+    """bench.py --sweep visits M in {1,2,4,8} and N in {1..4} unless told
+    otherwise; --sweep-M / --sweep-N take other replica and momentum counts
+    (the block-staged fused step's range, for instance)."""
+    sys.path.insert(0, ROOT)
+    import bench
+    monkeypatch.setattr("sys.argv", ["bench.py", "--sweep"])
+    a = bench.parse_args()
+    assert (a.sweep, a.sweep_M, a.sweep_N, a.sweep_log2n) == (True, "1,2,4,8", "1,2,3,4", "20,24,27,30")
+    monkeypatch.setattr("sys.argv", ["bench.py", "--sweep", "--sweep-M", "9,16,64", "--sweep-N", "3",
+                                     "--sweep-log2n", "26"])
+    a = bench.parse_args()
+    assert [int(v) for v in a.sweep_M.split(",")] == [9, 16, 64]
+    assert (a.sweep_N, a.sweep_log2n) == ("3", "26")
