@@ -3,8 +3,9 @@
 // that the one-pass diagnostics of stats_wide.cu share (up to kWideMaxM).
 //
 // A block owns a span of S consecutive elements of all M replicas; thread
-// (r, f) updates elements [4f, 4f + 4) of replica r (and [4(f + P), ...)
-// for M > 16, see wide_fused_vec) with update_state.  The
+// (r, f) updates elements [4f, 4f + 4) and [4(f + P), 4(f + P) + 4) of
+// replica r (one position above M = 32, see wide_fused_vec) with
+// update_state.  The
 // blocks are persistent and double-buffer their spans in shared memory: the
 // next span of every state and of the gradient is copied in with cp.async
 // while the current one is updated, so HBM traffic continues through the
@@ -21,8 +22,9 @@
 // A replica's row of a span is handled by P threads: P = 16 (M <= 16), 8
 // (M <= 64), 4 (M <= 128), 2 (M <= 256), so a block has M * P <= 512
 // threads (rounded up to whole warps; threads beyond M * P only take part
-// in the mean).  The fused step's rows are 64 elements (256 bytes) up to
-// M = 32 and 32 above; the one-pass diagnostics' rows are 16 P elements.
+// in the mean).  The fused step's rows are 128 elements (512 bytes) up to
+// M = 16, 64 up to 32 and 32 above; the one-pass diagnostics' rows are 16 P
+// elements.
 // Shared memory of the fused step: two span buffers (a tile per state and
 // the gradient tile) and S means per due state.
 #pragma once
@@ -166,12 +168,14 @@ __host__ __device__ constexpr int wide_buffer_floats(int M, int S) {
 }
 
 // Float4 positions per thread and row of the fused step's span (the
-// positions f and f + P): rows of 256 bytes up to M = 32 (S = 64).  With one
-// position and P = 8 (rows of 128 bytes) M = 24 and 32 ran at 4.8-4.9 TB/s
-// (Adam, N = 3), with two at 5.4, against 5.7-6.0 for M = 12-16.
-// Above 32 two positions made a span buffer so large (up to 96 KB) that
-// one block fitted per SM: M = 48 and 64 fell from 4.9-5.0 to 3.9-4.2 TB/s.
-constexpr int wide_fused_vec(int M) { return (M > 16 && M <= 32) ? 2 : 1; }
+// positions f and f + P): rows of 512 bytes up to M = 16 (S = 128) and 256
+// bytes for 17-32 (S = 64).  The row length sets the DRAM efficiency: with
+// one position, M = 24 and 32 (rows of 128 bytes) ran at 4.8-4.9 TB/s
+// (Adam, N = 3), with two at 5.4; M = 12 and 16 ran 3-10 % faster with
+// rows of 512 bytes than of 256.  Above 32 two positions made a span buffer
+// so large (up to 96 KB) that one block fitted per SM: M = 48 and 64 fell
+// from 4.9-5.0 to 3.9-4.2 TB/s.
+constexpr int wide_fused_vec(int M) { return M <= 32 ? 2 : 1; }
 
 // The fused step on spans of all replicas, persistent, double-buffered:
 // while a block updates span i from shared memory, span i + gridDim.x of
