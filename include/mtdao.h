@@ -244,8 +244,8 @@ int mtdao_set_params(mtdao_handle h, const float *x0_dev);
  * sync_mask: states to average over the replicas at the end of this same
  *   step (E_m[.] of Algorithm 1); usually the value of mtdao_sync_due.  The
  *   average is fused into the step's pass: it costs no extra HBM traffic for
- *   2 <= M <= 8 and M = 16; other M fall back to a separate averaging
- *   pass.
+ *   2 <= M <= 64 (a block stages a span of all replicas in shared memory
+ *   from M = 9); larger M fall back to a separate averaging pass.
  * With MTDAO_CLIP_GLOBAL_NORM a reduction pass over grads precedes the step.
  * With adopt_prev_v (the original ADOPT order) step 0 runs a separate pass
  * that writes v = g_0^2 and reads or writes nothing else, so u and x keep
@@ -289,9 +289,11 @@ int mtdao_step_host(mtdao_handle h, const void *grads_host, int32_t grad_dtype, 
  * h..M-1 (h = floor(M/2)), each in replica order; this returns s_0 bit for
  * bit when the replicas agree, and otherwise stays within a few roundings
  * of the largest replica value for any M (relative to the mean itself only
- * when the replicas do not cancel).  The fused average in mtdao_step and
- * mtdao_sync_stats use the same routine (identical bits).  mask 0 is a
- * no-op.
+ * when the replicas do not cancel).  Where that is NaN (the compensation
+ * meets an infinite value) the mean is the plain sum of the M values over
+ * M: +-Inf when they hold infinities of one sign, NaN otherwise.  The
+ * fused average in mtdao_step and mtdao_sync_stats use the same routine
+ * (identical bits).  mask 0 is a no-op.
  */
 int mtdao_sync(mtdao_handle h, uint32_t mask);
 
@@ -309,9 +311,10 @@ int mtdao_sync(mtdao_handle h, uint32_t mask);
  *                                                      sqrt([2+m] * [1]))
  * The averaged states are bit-identical to mtdao_sync's.  Sums are
  * fixed-order (bit-reproducible).  With M = 1 the states are left as they
- * are and only the diagnostics are written.  For M <= 8 the sums are
+ * are and only the diagnostics are written.  For M <= 64 the sums are
  * formed in the averaging pass itself (the sync's traffic, 8 M bytes per
- * element and state); for larger M each state takes two passes through a
+ * element and state; from M = 9 a block stages a span of all replicas in
+ * shared memory); for larger M each state takes two passes through a
  * library-owned [n_padded] fp32 scratch that holds the mean (about twice
  * the traffic), and (s_m - s_bar)^2 is summed as (s_m - s_0)^2 minus
  * M (s_bar - s_0)^2, in fp64.  Workspaces are allocated on the first call.
@@ -343,7 +346,7 @@ int mtdao_track_anchor(mtdao_handle h, uint32_t state_mask);
  * so cos(local, global) = [M+m] / sqrt([m] [2M]) and the relative change of
  * the averaged state over the round = sqrt([2M] / [2M+1]).  Call it before
  * the round's average of that state.  MTDAO_ERR_STATE if the state has no
- * anchor.  For M > 8 it takes two read-only passes through the scratch of
+ * anchor.  For M > 64 it takes two read-only passes through the scratch of
  * mtdao_sync_stats.
  */
 int mtdao_pseudo_grad_stats(mtdao_handle h, int32_t state, double *out_dev);
