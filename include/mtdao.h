@@ -316,8 +316,9 @@ int mtdao_sync(mtdao_handle h, uint32_t mask);
  * element and state; from M = 9 a block stages a span of all replicas in
  * shared memory); for larger M each state takes two passes through a
  * library-owned [n_padded] fp32 scratch that holds the mean (about twice
- * the traffic), and (s_m - s_bar)^2 is summed as (s_m - s_0)^2 minus
- * M (s_bar - s_0)^2, in fp64.  Workspaces are allocated on the first call.
+ * the traffic).  Every path forms (s_m - s_bar) against the fp32 mean it
+ * stores, sums a thread's elements in fp32 with Kahan compensation and
+ * adds the partial sums in fp64.  Workspaces are allocated on the first call.
  */
 int mtdao_sync_stats(mtdao_handle h, uint32_t mask, double *stats_dev);
 
