@@ -467,6 +467,49 @@ def test_sync_mean_brute_force_and_invariants():
         assert np.array_equal(a, again[k])      # idempotent
 
 
+def test_sync_mean_of_non_finite_values():
+    """The worker mean E_m[s] = sum_m s_m / M under IEEE arithmetic: a column
+    that holds infinities of one sign averages to that infinity, both signs
+    or a NaN give NaN, finite columns are the numpy mean.  (The GPU's
+    compensated mean falls back to this plain sum where it would give NaN.)"""
+    M, n = 4, 6
+    c = cfg("adam", (0.9,))
+    o = Oracle(c, M, n)
+    vals = np.arange(M * n, dtype=np.float64).reshape(M, n) / 7.0
+    vals[3, 0] = np.inf
+    vals[1, 1] = -np.inf
+    vals[0, 2], vals[3, 2] = np.inf, -np.inf
+    vals[2, 3] = np.nan
+    vals[:, 4] = -np.inf
+    o.x[:] = vals
+    o.sync(0b1)
+    got = o.states()["x"]
+    assert np.all(got == got[0:1]) or np.all(np.isnan(got) == np.isnan(got[0:1]))
+    row = got[0]
+    assert row[0] == np.inf and row[1] == -np.inf and np.isnan(row[2]) and np.isnan(row[3])
+    assert row[4] == -np.inf and row[5] == pytest.approx(vals[:, 5].mean(), rel=1e-15)
+
+
+@pytest.mark.parametrize("bad", [np.nan, np.inf, -np.inf])
+def test_adopt_original_ordering_step0_with_non_finite_gradient(bad):
+    """adopt_prev_v: step 0 only sets v = g_0^2, so a non-finite g_0 reaches
+    v alone (inf^2 = inf, nan^2 = nan); u stays 0 and x stays x_0."""
+    c = cfg("adopt", (0.9, 0.99), omega=(0.4, 0.5), beta2=0.9999, bias=False)
+    c["adopt_prev_v"] = True
+    M, n = 2, 8
+    x0 = np.linspace(-1.0, 1.0, n)
+    o = Oracle(c, M, n, x0=x0)
+    g0 = np.full((M, n), 0.5)
+    g0[1, 3] = bad
+    o.step(0, 0.1, g0)
+    assert np.all(o.u == 0) and np.all(o.x == x0[None, :])
+    v = o.v
+    assert (np.isnan(v[1, 3]) if np.isnan(bad) else v[1, 3] == np.inf)
+    mask = np.ones((M, n), bool)
+    mask[1, 3] = False
+    assert np.all(v[mask] == 0.25)
+
+
 def test_per_state_periods_counts():
     """H_x=64, H_u=H_v=16 over T=512 steps: x averaged 8 times, u and v 32."""
     c = cfg("adopt", (0.95, 0.999), beta2=0.9999, bias=False, px=64, pu=16, pv=16)
