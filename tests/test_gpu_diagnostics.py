@@ -74,6 +74,47 @@ def test_sync_stats_match_oracle_and_plain_sync(P, M):
         e.close()
 
 
+@pytest.mark.parametrize("M", [12, 40])
+def test_one_pass_diagnostics_over_many_spans(P, M):
+    """The one-pass diagnostics (9 <= M <= 64) run a persistent grid whose
+    blocks take many spans each, the next span's copy in flight while the
+    current one is summed: on a list of 2^21 elements every block walks
+    several spans.  Sums match the oracle's definitions, the averaged states
+    equal the plain average bit for bit, and the pseudo-gradient pass
+    matches its definition too."""
+    from oracle.oracle import pseudo_grad_stats
+    shapes = [1 << 21]
+    w = workload_dict(shapes, M, betas=(0.9, 0.99))
+    a = P.MTDAO(w["opt"], M, shapes)
+    b = P.MTDAO(w["opt"], M, shapes)
+    rng = np.random.default_rng(100 + M)
+    vals = _fill(a, rng, spread=0.05)
+    for s, arr in vals.items():
+        b.state_view(s).copy_(torch.from_numpy(arr).cuda())
+    mask = 0b111
+    stats = a.sync_stats(mask).cpu().numpy()
+    b.sync(mask)
+    torch.cuda.synchronize()
+    for row, s in zip(stats, range(3)):
+        ref = state_stats(vals[s].astype(np.float64))
+        err = np.abs(row - ref) / np.maximum(np.abs(ref), 1e-30)
+        assert np.all(err <= 1e-5), (s, err)
+    for s in range(3):
+        assert np.array_equal(a.state_view(s).cpu().numpy().view(np.uint32),
+                              b.state_view(s).cpu().numpy().view(np.uint32)), s
+    # pseudo-gradients of x against an anchor (its current value), after moving x
+    a.track_anchor(0b1)
+    anchor = a.state_view(0)[0].cpu().numpy().astype(np.float64)
+    moved = (a.state_view(0) + 0.01 * torch.randn((M, a.n_padded), device="cuda",
+                                                   generator=torch.Generator(device="cuda").manual_seed(M)))
+    a.state_view(0).copy_(moved)
+    got = a.pseudo_grad_stats(0).cpu().numpy()
+    cur = a.state_view(0).cpu().numpy().astype(np.float64)
+    np.testing.assert_allclose(got, pseudo_grad_stats(cur, anchor), rtol=1e-5)
+    a.close()
+    b.close()
+
+
 def test_sync_stats_cosine_and_variance_during_training(P):
     """After a few local steps from a common start, the cosine between each
     worker's momentum and the mean momentum is in (0, 1] and the variance
