@@ -30,10 +30,24 @@ def P():
 
 @pytest.mark.parametrize("M,N,H", POINTS)
 def test_sweep_point_parity(P, M, N, H):
-    from synth.device import DeviceInputs
     w = W.sweep_point(20, M, N, H)
     if N == 1 and H == 1:
         assert w["opt"]["omega"] == [1.0]
+    run_point(P, w, M, N, H)
+
+
+@pytest.mark.parametrize("M,N,H,base", [(16, 2, 4, "adopt"), (24, 3, 4, "adam"), (40, 1, 2, "sgdm")])
+def test_block_staged_fused_step_bf16_many_spans(P, M, N, H, base):
+    """bf16 gradients through the block-staged fused step with 2^20 elements
+    per replica: every persistent block walks many spans, each span's
+    gradient tile copied 8 bytes at a time while the previous one is used."""
+    w = W.sweep_point(20, M, N, H, base=base)
+    w["grad_dtype"] = "bf16"
+    run_point(P, w, M, N, H)
+
+
+def run_point(P, w, M, N, H):
+    from synth.device import DeviceInputs
     lay = W.layout(w["shapes"])
     opt, T = w["opt"], w["T"]
     eng = P.MTDAO(opt, M, w["shapes"])
