@@ -74,16 +74,17 @@ def test_sync_stats_match_oracle_and_plain_sync(P, M):
         e.close()
 
 
-@pytest.mark.parametrize("M", [12, 40])
+@pytest.mark.parametrize("M", [4, 12, 40])
 def test_one_pass_diagnostics_over_many_spans(P, M):
-    """The one-pass diagnostics (9 <= M <= 64) run a persistent grid whose
-    blocks take many spans each, the next span's copy in flight while the
-    current one is summed: on a list of 2^21 elements every block walks
-    several spans.  Sums match the oracle's definitions, the averaged states
-    equal the plain average bit for bit, and the pseudo-gradient pass
-    matches its definition too."""
+    """Large lists: the one-pass diagnostics for 9 <= M <= 64 run a
+    persistent grid whose blocks take many spans each (2^21 elements), the
+    next span's copy in flight while the current one is summed; for M = 4
+    the sync diagnostics run 264 tile blocks per state, so the finalize adds
+    runs of block rows per thread, and the pseudo-gradient pass runs its
+    whole persistent grid.  Sums match the oracle's definitions, the averaged
+    states equal the plain average bit for bit."""
     from oracle.oracle import pseudo_grad_stats
-    shapes = [1 << 21]
+    shapes = [1 << 25, 1 << 20] if M <= 8 else [1 << 21]
     w = workload_dict(shapes, M, betas=(0.9, 0.99))
     a = P.MTDAO(w["opt"], M, shapes)
     b = P.MTDAO(w["opt"], M, shapes)
