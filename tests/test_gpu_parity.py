@@ -163,6 +163,39 @@ def test_grad_sqnorm(P, gdt):
     eng.close()
 
 
+@pytest.mark.parametrize("M,gdt", [(4, "f32"), (8, "bf16")])
+def test_grad_sqnorm_and_nonfinite_count_at_scale(P, M, gdt):
+    """2^26 elements per replica: every thread of the norm kernels walks
+    hundreds of strided positions (16-byte loads: 4 f32 or 8 bf16 values).
+    The sum of squares matches an fp64 sum taken by torch on the device
+    (1e-6 relative, as the oracle's norm tests) and is reproducible; the
+    non-finite count finds planted values exactly."""
+    from synth.device import DeviceInputs
+    shapes = [1 << 26]
+    w = workload_dict(shapes, M, sigma=0.5, gdt=gdt)
+    lay = W.layout(shapes)
+    g = DeviceInputs(w, lay, SEED_G, SEED_I).grads(0)
+    eng = P.MTDAO(w["opt"], M, shapes)
+    dt = P.BF16 if gdt == "bf16" else P.F32
+    out = torch.zeros(M, dtype=torch.float64, device="cuda")
+    again = torch.zeros_like(out)
+    P.mtdao_grad_sqnorm(eng.h, g.data_ptr(), dt, out.data_ptr())
+    P.mtdao_grad_sqnorm(eng.h, g.data_ptr(), dt, again.data_ptr())
+    expect = (g.double() ** 2).sum(dim=1)
+    assert torch.equal(out, again)
+    assert float(((out - expect).abs() / expect).max()) < 1e-6
+    g[M - 1, 12345] = float("nan")
+    g[0, (1 << 26) - 3] = float("inf")
+    g[0, 7] = float("-inf")
+    cnt = torch.zeros(M, dtype=torch.float64, device="cuda")
+    P.mtdao_grad_nonfinite(eng.h, g.data_ptr(), dt, cnt.data_ptr())
+    want = [0.0] * M
+    want[0] += 2
+    want[M - 1] += 1
+    assert cnt.cpu().tolist() == want
+    eng.close()
+
+
 @pytest.mark.parametrize("gdt", ["f32", "bf16"])
 def test_grad_sqnorm_extreme_range(P, gdt):
     """Sums of squares whose terms leave fp32's range: replica 0 holds a few
